@@ -1,0 +1,201 @@
+"""CPU oracle for the structure-aware banded LU dispatch (Lujan & Edelman, HPEC 2025).
+
+TEST INFRASTRUCTURE ONLY.  The functions here are the independent reference the
+CUDA path is checked against.  Only the test suite, ``__graft_entry__.smoke()``
+and the benchmark's CPU-baseline leg may import this package; the CUDA library
+and its Python binding never do.
+
+The arithmetic lives in ``bandlu_oracle.c`` (plain C, IEEE binary64, built with
+``-ffp-contract=off``); this module compiles it with gcc on first use and wraps
+it with ctypes over numpy arrays.
+
+Layouts: ``A`` is a dense row-major ``(n, lda)`` float64 array (only the first
+``n`` columns are the matrix); ``AB`` is LAPACK band storage, column-major
+``ldab x n``, held here as a numpy array of shape ``(n, ldab)`` whose row ``j``
+is band column ``j`` (so ``AB[j, r]`` is ``AB(r, j)``); ``ipiv`` is 1-based.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "bandlu_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "liboracle_bandlu.so")
+_lock = threading.Lock()
+_lib = None
+
+CFLAGS = ["-O2", "-fPIC", "-shared", "-std=gnu11", "-ffp-contract=off", "-fno-fast-math"]
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc into ``oracle/_build``; returns the .so path."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    subprocess.run(["gcc", *CFLAGS, "-o", tmp, _SRC, "-lm"], check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        # A mutation test points this at a deliberately broken build of the oracle to show that
+        # the pins catch the mistake; normal use leaves it unset.
+        path = os.environ.get("BANDLU_ORACLE_LIB") or build()
+        lib = ctypes.CDLL(path)
+        i64, i32, dp, ip = ctypes.c_int64, ctypes.c_int, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)
+        i64p = ctypes.POINTER(ctypes.c_int64)
+        lib.oracle_detect_bandwidth.argtypes = [dp, i64, i64, ip, ip]
+        lib.oracle_dense_to_band.argtypes = [dp, i64, i64, i32, i32, dp, i64]
+        lib.oracle_band_to_dense.argtypes = [i64, i32, i32, dp, i64, dp, i64]
+        lib.oracle_gbtrf.argtypes = [i64, i32, i32, dp, i64, ip, i64p]
+        lib.oracle_getrf_dense.argtypes = [i64, dp, i64, ip]
+        lib.oracle_band_residual.argtypes = [i64, i32, i32, dp, i64, dp, i64, ip, dp, dp]
+        lib.oracle_band_residual.restype = ctypes.c_double
+        lib.oracle_is_banded.argtypes = [i64, i32, i32, i64]
+        lib.oracle_dispatch_lu_batched.argtypes = [dp, i64, i64, i64, i64, dp, i64, i64, ip, i64, ip, ip, ip, ip]
+        lib.oracle_dispatch_lu_batched.restype = None
+        _lib = lib
+        return lib
+
+
+def _dptr(a: np.ndarray):
+    assert a.dtype == np.float64 and a.flags.c_contiguous
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_double))
+
+
+def _iptr(a: np.ndarray):
+    assert a.dtype == np.int32 and a.flags.c_contiguous
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
+
+
+def _dense(A: np.ndarray):
+    A = np.ascontiguousarray(A, dtype=np.float64)
+    n, lda = A.shape[0], A.shape[1]
+    assert lda >= n
+    return A, n, lda
+
+
+def ldab_for(kl: int, ku: int) -> int:
+    """Height of LAPACK band storage with room for pivoting fill: 2*kl+ku+1."""
+    return 2 * kl + ku + 1
+
+
+def detect_bandwidth(A: np.ndarray) -> tuple[int, int]:
+    """(kl, ku) of the n x n row-major matrix held in ``A[:, :n]``."""
+    A, n, lda = _dense(A)
+    kl, ku = ctypes.c_int(), ctypes.c_int()
+    rc = _load().oracle_detect_bandwidth(_dptr(A), n, max(lda, 1), ctypes.byref(kl), ctypes.byref(ku))
+    if rc != 0:
+        raise ValueError("oracle_detect_bandwidth: bad argument")
+    return kl.value, ku.value
+
+
+def dense_to_band(A: np.ndarray, kl: int, ku: int, ldab: int | None = None) -> np.ndarray:
+    """Band storage of A as an (n, ldab) array: ``AB[j, kl+ku+i-j] = A[i, j]``."""
+    A, n, lda = _dense(A)
+    ldab = ldab_for(kl, ku) if ldab is None else ldab
+    AB = np.empty((n, ldab), dtype=np.float64)
+    rc = _load().oracle_dense_to_band(_dptr(A), n, max(lda, 1), kl, ku, _dptr(AB), ldab)
+    if rc != 0:
+        raise ValueError("oracle_dense_to_band: bad argument")
+    return AB
+
+
+def band_to_dense(AB: np.ndarray, kl: int, ku: int) -> np.ndarray:
+    AB = np.ascontiguousarray(AB, dtype=np.float64)
+    n, ldab = AB.shape
+    A = np.empty((n, n), dtype=np.float64)
+    rc = _load().oracle_band_to_dense(n, kl, ku, _dptr(AB), ldab, _dptr(A), max(n, 1))
+    if rc != 0:
+        raise ValueError("oracle_band_to_dense: bad argument")
+    return A
+
+
+def gbtrf(AB: np.ndarray, kl: int, ku: int) -> tuple[np.ndarray, np.ndarray, int, int]:
+    """Factor a copy of the band; returns (AB_factored, ipiv (1-based int32), info, flops)."""
+    AB = np.array(AB, dtype=np.float64, order="C", copy=True)
+    n, ldab = AB.shape
+    ipiv = np.zeros(n, dtype=np.int32)
+    fl = ctypes.c_int64()
+    info = _load().oracle_gbtrf(n, kl, ku, _dptr(AB), ldab, _iptr(ipiv), ctypes.byref(fl))
+    if info < 0:
+        raise ValueError("oracle_gbtrf: bad argument")
+    return AB, ipiv, info, fl.value
+
+
+def getrf_dense(A: np.ndarray) -> tuple[np.ndarray, np.ndarray, int]:
+    """Dense LU of a copy of A (row-major), interchanges over columns j..n-1 only."""
+    A = np.array(A, dtype=np.float64, order="C", copy=True)
+    n, lda = A.shape
+    ipiv = np.zeros(n, dtype=np.int32)
+    info = _load().oracle_getrf_dense(n, _dptr(A), max(lda, 1), _iptr(ipiv))
+    if info < 0:
+        raise ValueError("oracle_getrf_dense: bad argument")
+    return A, ipiv, info
+
+
+def band_residual(A: np.ndarray, ABf: np.ndarray, ipiv: np.ndarray, kl: int, ku: int) -> tuple[float, float]:
+    """(||A - P0 L0 ... U||_inf, ||A||_inf) computed in band form."""
+    A, n, lda = _dense(A)
+    ABf = np.ascontiguousarray(ABf, dtype=np.float64)
+    ipiv = np.ascontiguousarray(ipiv, dtype=np.int32)
+    assert ABf.shape[0] == n
+    W = np.empty(max(n * (2 * kl + ku + 1), 1), dtype=np.float64)
+    an = ctypes.c_double()
+    r = _load().oracle_band_residual(n, kl, ku, _dptr(A), max(lda, 1), _dptr(ABf), ABf.shape[1],
+                                     _iptr(ipiv), _dptr(W), ctypes.byref(an))
+    return r, an.value
+
+
+def backward_error(A: np.ndarray, ABf: np.ndarray, ipiv: np.ndarray, kl: int, ku: int,
+                   eps: float = 2.0 ** -53) -> float:
+    """||A - P L U||_inf / (n * eps * ||A||_inf); eps defaults to the unit roundoff."""
+    n = A.shape[0]
+    r, an = band_residual(A, ABf, ipiv, kl, ku)
+    if n == 0 or an == 0.0:
+        return 0.0 if r == 0.0 else float("inf")
+    return r / (n * eps * an)
+
+
+def is_banded(n: int, kl: int, ku: int, ldab: int) -> bool:
+    """The dispatch predicate: the speedup constraint (Eq. su-con) and the storage capacity."""
+    return bool(_load().oracle_is_banded(n, kl, ku, ldab))
+
+
+def dispatch_lu_batched(A: np.ndarray, ldab: int):
+    """Batched dispatch over A of shape (batch, n, lda).
+
+    Returns dict with AB (batch, n, ldab), ipiv (batch, n), kl, ku, info, status
+    (0 = factored, 1 = declined by the predicate).
+    """
+    A = np.ascontiguousarray(A, dtype=np.float64)
+    batch, n, lda = A.shape
+    AB = np.zeros((batch, n, ldab), dtype=np.float64)
+    ipiv = np.zeros((batch, n), dtype=np.int32)
+    kl = np.zeros(batch, dtype=np.int32)
+    ku = np.zeros(batch, dtype=np.int32)
+    info = np.zeros(batch, dtype=np.int32)
+    status = np.zeros(batch, dtype=np.int32)
+    _load().oracle_dispatch_lu_batched(_dptr(A), n, max(lda, 1), n * lda, batch, _dptr(AB), ldab, n * ldab,
+                                       _iptr(ipiv), n, _iptr(kl), _iptr(ku), _iptr(info), _iptr(status))
+    return dict(AB=AB, ipiv=ipiv, kl=kl, ku=ku, info=info, status=status)
+
+
+def dispatch_lu(A: np.ndarray, ldab: int):
+    """Single-matrix dispatch (the batched routine with batch 1)."""
+    A = np.ascontiguousarray(A, dtype=np.float64)
+    r = dispatch_lu_batched(A[None], ldab)
+    return dict(AB=r["AB"][0], ipiv=r["ipiv"][0], kl=int(r["kl"][0]), ku=int(r["ku"][0]),
+                info=int(r["info"][0]), status=int(r["status"][0]))

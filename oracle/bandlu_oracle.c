@@ -1,0 +1,330 @@
+/*
+ * bandlu_oracle.c -- plain, slow, single-threaded CPU oracle for the
+ * structure-aware banded LU dispatch of Lujan & Edelman, "When Structure is
+ * Silent: Opportunities for Algorithmic Dispatch in Linear Algebra" (HPEC 2025).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the independent reference that the
+ * CUDA path is checked against.  Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline leg may load it.  The CUDA library never links,
+ * includes or calls anything here, and nothing here includes the library's
+ * headers.
+ *
+ * Arithmetic is IEEE binary64, compiled with -ffp-contract=off so that the
+ * only fused multiply-adds are the explicit fma() calls written below.
+ *
+ * Layouts (0-based everywhere in this file):
+ *   A   dense, ROW-major, n x n, leading dimension lda >= n:  A(i,j) = A[i*lda + j]
+ *   AB  LAPACK band storage, COLUMN-major, ldab x n, kv = kl + ku,
+ *       ldab >= 2*kl + ku + 1:  A(i,j) lives at AB(kv + i - j, j) = AB[(kv+i-j) + j*ldab]
+ *       rows 0..kl-1 are the fill rows that row interchanges spill into.
+ *   ipiv 1-based pivot rows (LAPACK convention): row j was interchanged with row ipiv[j]-1.
+ *
+ * Parity status of each function (what pins it is listed in the test suite):
+ *   oracle_detect_bandwidth   pinned (definition; istril/istriu characterisation; special cases)
+ *   oracle_dense_to_band      pinned (round trip; a library band solver consumes the layout)
+ *   oracle_gbtrf              pinned (LAPACK dgbtrf; dense LU equivalence; closed form; backward error)
+ *   oracle_getrf_dense        pinned (LAPACK dgetrf; exact rational elimination)
+ *   oracle_band_residual      pinned (dense reconstruction with a library matmul)
+ *   oracle_is_banded          pinned (the worked cases of the speedup constraint, Eq. su-con)
+ */
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+/* A double counts as a nonzero element iff it compares unequal to 0.0 under
+ * IEEE rules: -0.0 is zero; NaN, +-Inf and subnormals are nonzero.  This is
+ * the element inspection the paper's Listing 1 performs through istril/istriu
+ * (Sec. I-C) and that banded_structure performs in Listing 2 (Sec. IV). */
+static int is_nonzero(double x) { return x != 0.0; }
+
+/*
+ * Structure identification, cost I(N) ~ O(N^2) (Sec. III-A, Eq. IC-N2; step 1
+ * of the strategy in Sec. II-A).  Definition: kl is the largest i-j over the
+ * nonzero elements of A, ku the largest j-i, both clamped below at 0.  Every
+ * element is inspected.  Returns 0, or -1 on a bad argument.
+ */
+int oracle_detect_bandwidth(const double *A, int64_t n, int64_t lda, int *kl, int *ku)
+{
+    if (n < 0 || lda < (n > 1 ? n : 1) || !kl || !ku) return -1;
+    int64_t best_l = 0, best_u = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        for (int64_t j = 0; j < n; ++j) {
+            if (is_nonzero(A[i * lda + j])) {
+                if (i - j > best_l) best_l = i - j;
+                if (j - i > best_u) best_u = j - i;
+            }
+        }
+    }
+    *kl = (int)best_l;
+    *ku = (int)best_u;
+    return 0;
+}
+
+/*
+ * Format conversion, cost C(N) (Sec. III-A, Eq. IC-N2; step 2 of Sec. II-A;
+ * BandedMatrix(A) in Listing 2).  Target is LAPACK's xGBTRF band storage
+ * (Sec. I-A cites xGBTRF): AB(kv+i-j, j) = A(i,j) for max(0,j-ku) <= i <= min(n-1,j+kl).
+ * Every other entry of AB (fill rows 0..kl-1, the corner triangles and rows
+ * beyond 2kl+ku) is set to +0.0.  A is not modified.
+ */
+int oracle_dense_to_band(const double *A, int64_t n, int64_t lda, int kl, int ku,
+                         double *AB, int64_t ldab)
+{
+    if (n < 0 || kl < 0 || ku < 0 || lda < (n > 1 ? n : 1) || ldab < 2 * (int64_t)kl + ku + 1) return -1;
+    int64_t kv = (int64_t)kl + ku;
+    for (int64_t j = 0; j < n; ++j) {
+        for (int64_t r = 0; r < ldab; ++r) AB[r + j * ldab] = 0.0;
+        int64_t i0 = j - ku > 0 ? j - ku : 0;
+        int64_t i1 = j + kl < n - 1 ? j + kl : n - 1;
+        for (int64_t i = i0; i <= i1; ++i) AB[(kv + i - j) + j * ldab] = A[i * lda + j];
+    }
+    return 0;
+}
+
+/* Inverse of the conversion for the band rows kl..2kl+ku (test helper):
+ * writes the dense matrix with zeros outside the band. */
+int oracle_band_to_dense(int64_t n, int kl, int ku, const double *AB, int64_t ldab,
+                         double *A, int64_t lda)
+{
+    if (n < 0 || kl < 0 || ku < 0 || lda < (n > 1 ? n : 1) || ldab < 2 * (int64_t)kl + ku + 1) return -1;
+    int64_t kv = (int64_t)kl + ku;
+    for (int64_t i = 0; i < n; ++i)
+        for (int64_t j = 0; j < n; ++j) A[i * lda + j] = 0.0;
+    for (int64_t j = 0; j < n; ++j) {
+        int64_t i0 = j - ku > 0 ? j - ku : 0;
+        int64_t i1 = j + kl < n - 1 ? j + kl : n - 1;
+        for (int64_t i = i0; i <= i1; ++i) A[i * lda + j] = AB[(kv + i - j) + j * ldab];
+    }
+    return 0;
+}
+
+/*
+ * Banded LU with partial pivoting, cost f(N) ~ O(N*P*Q) (Sec. III-A,
+ * Eq. S-N-N3; step 3 of Sec. II-A; lu(A_banded) -> DGBTRF in Listing 2).
+ *
+ * Unblocked right-looking Gaussian elimination on the band, in the order the
+ * elimination is defined:  for each column j, pick the pivot as the FIRST
+ * element of largest magnitude among rows j..j+km (km = min(kl, n-1-j));
+ * interchange rows j and the pivot row over the columns that the upper factor
+ * can reach so far (j..ju); scale the km subdiagonal entries by the reciprocal
+ * of the pivot; subtract the rank-1 product from the trailing window.  An
+ * exactly zero pivot records info = j+1 (first such column) and the column is
+ * skipped; elimination continues, so info > 0 is not an error.
+ *
+ * On exit AB holds U in rows 0..kv (upper bandwidth kv = kl+ku) and the
+ * multipliers of column j in rows kv+1..kv+km of column j, unpermuted by later
+ * interchanges (A = P_0 L_0 P_1 L_1 ... P_{n-1} L_{n-1} U).
+ *
+ * The fill rows 0..kl-1 are cleared first, so they need not be zero on entry.
+ * The trailing update skips a column whose pivot-row entry u is exactly zero;
+ * the skipped operation is x - l*0.  Updates are fma(-l, u, x), one rounding.
+ *
+ * *flops (optional) receives sum_j [1 + km + 2*km*(ju_j - j)] over the columns
+ * with a nonzero pivot: one reciprocal, km scalings, and the nominal rank-1
+ * update of the km x (ju_j - j) window.  Returns info (>= 0), or -1 on a bad argument.
+ */
+int oracle_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int64_t *flops)
+{
+    if (n < 0 || kl < 0 || ku < 0 || ldab < 2 * (int64_t)kl + ku + 1) return -1;
+    const int64_t kv = (int64_t)kl + ku;
+#define AB_(r, c) AB[(r) + (c) * ldab]
+    for (int64_t c = 0; c < n; ++c)
+        for (int64_t r = 0; r < kl; ++r) AB_(r, c) = 0.0;
+    int info = 0;
+    int64_t ju = 0;
+    int64_t fl = 0;
+    for (int64_t j = 0; j < n; ++j) {
+        int64_t km = (int64_t)kl < n - 1 - j ? (int64_t)kl : n - 1 - j;
+        /* pivot search: first index of the largest |AB(kv+t, j)|, t = 0..km */
+        int64_t p = 0;
+        double best = fabs(AB_(kv, j));
+        for (int64_t t = 1; t <= km; ++t) {
+            double v = fabs(AB_(kv + t, j));
+            if (v > best) { best = v; p = t; }
+        }
+        ipiv[j] = (int)(j + p + 1);
+        if (AB_(kv + p, j) != 0.0) {
+            int64_t reach = j + ku + p < n - 1 ? j + ku + p : n - 1;
+            if (reach > ju) ju = reach;
+            if (p != 0) {
+                /* row j+p and row j, columns j..ju: element (i, c) is at AB(kv+i-c, c) */
+                for (int64_t c = j; c <= ju; ++c) {
+                    double t0 = AB_(kv + j - c, c);
+                    AB_(kv + j - c, c) = AB_(kv + j + p - c, c);
+                    AB_(kv + j + p - c, c) = t0;
+                }
+            }
+            if (km > 0) {
+                double rcp = 1.0 / AB_(kv, j);
+                for (int64_t t = 1; t <= km; ++t) AB_(kv + t, j) *= rcp;
+                for (int64_t c = j + 1; c <= ju; ++c) {
+                    double u = AB_(kv + j - c, c); /* U(j, c) */
+                    if (u != 0.0) {
+                        for (int64_t t = 1; t <= km; ++t) {
+                            /* element (j+t, c) */
+                            AB_(kv + j + t - c, c) = fma(-AB_(kv + t, j), u, AB_(kv + j + t - c, c));
+                        }
+                    }
+                }
+            }
+            fl += 1 + km + 2 * km * (ju - j);
+        } else if (info == 0) {
+            info = (int)(j + 1);
+        }
+    }
+#undef AB_
+    if (flops) *flops = fl;
+    return info;
+}
+
+/*
+ * The generic algorithm F(N) ~ O(N^3) of Sec. III-A (Eq. D-N3; DGETRF in
+ * Listing 2), written as plain dense Gaussian elimination on the row-major
+ * matrix with the same pivot rule, reciprocal scaling, fma update and
+ * zero-u skip as oracle_gbtrf, and with the interchange applied to columns
+ * j..n-1 only (multipliers stay where they were computed, the same
+ * P_0 L_0 P_1 L_1 ... U form).  With no band bookkeeping at all, it serves as
+ * the brute-force check of oracle_gbtrf.  Returns info.
+ */
+int oracle_getrf_dense(int64_t n, double *A, int64_t lda, int *ipiv)
+{
+    if (n < 0 || lda < (n > 1 ? n : 1)) return -1;
+    int info = 0;
+    for (int64_t j = 0; j < n; ++j) {
+        int64_t p = j;
+        double best = fabs(A[j * lda + j]);
+        for (int64_t i = j + 1; i < n; ++i) {
+            double v = fabs(A[i * lda + j]);
+            if (v > best) { best = v; p = i; }
+        }
+        ipiv[j] = (int)(p + 1);
+        if (A[p * lda + j] != 0.0) {
+            if (p != j) {
+                for (int64_t c = j; c < n; ++c) {
+                    double t0 = A[j * lda + c];
+                    A[j * lda + c] = A[p * lda + c];
+                    A[p * lda + c] = t0;
+                }
+            }
+            if (j < n - 1) {
+                double rcp = 1.0 / A[j * lda + j];
+                for (int64_t i = j + 1; i < n; ++i) A[i * lda + j] *= rcp;
+                for (int64_t c = j + 1; c < n; ++c) {
+                    double u = A[j * lda + c];
+                    if (u != 0.0) {
+                        for (int64_t i = j + 1; i < n; ++i)
+                            A[i * lda + c] = fma(-A[i * lda + j], u, A[i * lda + c]);
+                    }
+                }
+            }
+        } else if (info == 0) {
+            info = (int)(j + 1);
+        }
+    }
+    return info;
+}
+
+/*
+ * Backward error of a band factorisation: returns ||A - P_0 L_0 ... P_{n-1} L_{n-1} U||_inf
+ * (max row sum) and writes ||A||_inf to *anorm.  The product is rebuilt from
+ * U by applying, for j = n-1 down to 0, first L_j (row j+t += l_{j+t,j} * row j)
+ * and then the interchange of rows j and ipiv[j]-1.  Rows j..j+kl of every
+ * intermediate product have nonzeros only in columns j..j+kv, so the rebuild
+ * is held in a band of lower width kl and upper width kv: the work array W
+ * must hold n*(2*kl+ku+1) doubles.  A is the original dense row-major matrix.
+ */
+double oracle_band_residual(int64_t n, int kl, int ku, const double *A, int64_t lda,
+                            const double *AB, int64_t ldab, const int *ipiv,
+                            double *W, double *anorm)
+{
+    const int64_t kv = (int64_t)kl + ku;
+    const int64_t w = (int64_t)kl + kv + 1; /* row i of M holds columns i-kl .. i+kv */
+#define M_(i, c) W[(i) * w + ((c) - (i) + kl)]
+    for (int64_t i = 0; i < n * w; ++i) W[i] = 0.0;
+    for (int64_t i = 0; i < n; ++i) {
+        int64_t c1 = i + kv < n - 1 ? i + kv : n - 1;
+        for (int64_t c = i; c <= c1; ++c) M_(i, c) = AB[(kv + i - c) + c * ldab];
+    }
+    for (int64_t j = n - 1; j >= 0; --j) {
+        int64_t km = (int64_t)kl < n - 1 - j ? (int64_t)kl : n - 1 - j;
+        int64_t c1 = j + kv < n - 1 ? j + kv : n - 1;
+        for (int64_t t = 1; t <= km; ++t) {
+            double l = AB[(kv + t) + j * ldab];
+            for (int64_t c = j; c <= c1; ++c) M_(j + t, c) += l * M_(j, c);
+        }
+        int64_t p = (int64_t)ipiv[j] - 1;
+        if (p != j) {
+            for (int64_t c = j; c <= c1; ++c) {
+                double t0 = M_(j, c);
+                M_(j, c) = M_(p, c);
+                M_(p, c) = t0;
+            }
+        }
+    }
+    double rnorm = 0.0, an = 0.0;
+    for (int64_t i = 0; i < n; ++i) {
+        double rs = 0.0, as = 0.0;
+        int64_t c0 = i - kl > 0 ? i - kl : 0;
+        int64_t c1 = i + kv < n - 1 ? i + kv : n - 1;
+        for (int64_t c = c0; c <= c1; ++c) {
+            double a = (c - i <= ku) ? A[i * lda + c] : 0.0;
+            rs += fabs(a - M_(i, c));
+            as += fabs(a);
+        }
+        if (rs > rnorm) rnorm = rs;
+        if (as > an) an = as;
+    }
+#undef M_
+    if (anorm) *anorm = an;
+    return rnorm;
+}
+
+/*
+ * The dispatch predicate (banded_structure in Listing 2, Sec. IV): the band
+ * path is taken iff the speedup constraint I(N) + C(N) + f(N) < F(N) of
+ * Eq. su-con (Sec. II-B) holds with the operation counts
+ *   I(N) = n^2                       one inspection per element (Eq. IC-N2)
+ *   C(N) = n*(kl+ku+1)               one copy per band element (Eq. IC-N2)
+ *   f(N) = n*kl*(2*(kl+ku)+1)        banded LU, worst-case fill (Eq. S-N-N3)
+ *   F(N) = 2*n^3/3                   dense LU (Eq. D-N3)
+ * evaluated exactly as 3*(I+C+f) < 2*n^3 in 128-bit integers, and the caller's
+ * band storage can hold the factors (2*kl+ku+1 <= ldab).  Returns 1 or 0.
+ */
+int oracle_is_banded(int64_t n, int kl, int ku, int64_t ldab)
+{
+    if (2 * (int64_t)kl + ku + 1 > ldab) return 0;
+    __int128 N = n, L = kl, U = ku;
+    __int128 I = N * N;
+    __int128 C = N * (L + U + 1);
+    __int128 f = N * L * (2 * (L + U) + 1);
+    __int128 F3 = 2 * N * N * N; /* 3*F */
+    return 3 * (I + C + f) < F3 ? 1 : 0;
+}
+
+/*
+ * The whole strategy of Sec. II-A for one matrix (Listing 2 without the dense
+ * branch): identify, decide, convert, factor.  Returns 0 when the band path
+ * ran (info in *info), 1 when the predicate declined (AB, ipiv untouched).
+ */
+int oracle_dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab,
+                       int *ipiv, int *kl, int *ku, int *info)
+{
+    if (oracle_detect_bandwidth(A, n, lda, kl, ku) != 0) return -1;
+    if (!oracle_is_banded(n, *kl, *ku, ldab)) return 1;
+    oracle_dense_to_band(A, n, lda, *kl, *ku, AB, ldab);
+    *info = oracle_gbtrf(n, *kl, *ku, AB, ldab, ipiv, 0);
+    return 0;
+}
+
+/* The same strategy over a batch of independent matrices, one after another:
+ * matrix b at A + b*strideA, AB + b*strideAB, ipiv + b*strideP. */
+void oracle_dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch,
+                                double *AB, int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP,
+                                int *kl, int *ku, int *info, int *status)
+{
+    for (int64_t b = 0; b < batch; ++b) {
+        info[b] = 0;
+        status[b] = oracle_dispatch_lu(A + b * strideA, n, lda, AB + b * strideAB, ldab,
+                                       ipiv + b * strideP, kl + b, ku + b, info + b);
+    }
+}

@@ -1,0 +1,59 @@
+"""The oracle's pins must catch plausible mistakes.
+
+Each case below plants one mistake in a copy of the oracle's C source (on the CPU,
+never in the CUDA path), builds it, and runs the pin suite against the broken build
+in a subprocess.  The suite must fail for every mutant.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "bandlu_oracle.c")
+
+# (name, text to replace, replacement): each text occurs in the source; the first occurrence is replaced
+MUTANTS = [
+    ("ipiv_zero_based", "ipiv[j] = (int)(j + p + 1);\n        if (AB_", "ipiv[j] = (int)(j + p);\n        if (AB_"),
+    ("last_max_tie_break", "if (v > best) { best = v; p = t; }", "if (v >= best) { best = v; p = t; }"),
+    ("update_sign", "fma(-AB_(kv + t, j), u,", "fma(AB_(kv + t, j), u,"),
+    ("short_swap_range", "for (int64_t c = j; c <= ju; ++c) {", "for (int64_t c = j; c < ju; ++c) {"),
+    ("km_not_clamped", "int64_t km = (int64_t)kl < n - 1 - j ? (int64_t)kl : n - 1 - j;\n        /* pivot",
+     "int64_t km = (int64_t)kl;\n        /* pivot"),
+    ("reach_ignores_pivot_row", "int64_t reach = j + ku + p < n - 1 ? j + ku + p : n - 1;",
+     "int64_t reach = j + ku < n - 1 ? j + ku : n - 1;"),
+    ("divide_instead_of_reciprocal", "for (int64_t t = 1; t <= km; ++t) AB_(kv + t, j) *= rcp;",
+     "for (int64_t t = 1; t <= km; ++t) AB_(kv + t, j) /= AB_(kv, j);"),
+    ("pivot_search_misses_last_row", "for (int64_t t = 1; t <= km; ++t) {\n            double v",
+     "for (int64_t t = 1; t < km; ++t) {\n            double v"),
+    ("detect_lower_upper_swapped", "if (i - j > best_l) best_l = i - j;", "if (j - i > best_l) best_l = j - i;"),
+    ("convert_drops_last_subdiagonal", "int64_t i1 = j + kl < n - 1 ? j + kl : n - 1;\n        for (int64_t i = i0; i <= i1; ++i) AB[(kv + i - j) + j * ldab] = A",
+     "int64_t i1 = j + kl - 1 < n - 1 ? j + kl - 1 : n - 1;\n        for (int64_t i = i0; i <= i1; ++i) AB[(kv + i - j) + j * ldab] = A"),
+    ("residual_drops_interchange", "if (p != j) {\n            for (int64_t c = j; c <= c1; ++c) {",
+     "if (0) {\n            for (int64_t c = j; c <= c1; ++c) {"),
+    ("fill_rows_not_cleared", "for (int64_t r = 0; r < kl; ++r) AB_(r, c) = 0.0;", "for (int64_t r = 0; r < 0; ++r) AB_(r, c) = 0.0;"),
+    ("info_reports_last_zero_pivot", "} else if (info == 0) {\n            info = (int)(j + 1);\n        }\n    }\n#undef AB_",
+     "} else {\n            info = (int)(j + 1);\n        }\n    }\n#undef AB_"),
+    ("predicate_drops_conversion_cost", "return 3 * (I + C + f) < F3 ? 1 : 0;", "return 3 * (I + f) < F3 ? 1 : 0;"),
+    ("flops_drop_reciprocal", "fl += 1 + km + 2 * km * (ju - j);", "fl += km + 2 * km * (ju - j);"),
+    ("dense_lu_swaps_whole_row", "for (int64_t c = j; c < n; ++c) {\n                    double t0 = A[j * lda + c];",
+     "for (int64_t c = 0; c < n; ++c) {\n                    double t0 = A[j * lda + c];"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_mutant(tmp_path, name, old, new):
+    src = open(SRC).read()
+    assert old in src, f"mutation site for {name} not found"
+    mutated = src.replace(old, new, 1)
+    c_path = tmp_path / "mutant.c"
+    so_path = tmp_path / "libmutant.so"
+    c_path.write_text(mutated)
+    sys.path.insert(0, ROOT)
+    import oracle
+    subprocess.run(["gcc", *oracle.CFLAGS, "-o", str(so_path), str(c_path), "-lm"], check=True)
+    env = dict(os.environ, BANDLU_ORACLE_LIB=str(so_path))
+    r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle.py"), "-x", "-q"],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"pins did not catch mutant {name}:\n{r.stdout[-2000:]}"
