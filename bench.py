@@ -1,0 +1,366 @@
+"""Benchmark of the structure-aware banded LU dispatch on GB300.
+
+One step = one dispatch_lu call (detect the bandwidths of the dense matrix,
+decide, convert to band storage, factor the band) on the synthetic
+n = 4096, kl = ku = 16 fp64 matrix (uniform[-1,1] band, no diagonal boost, so
+partial pivoting swaps rows), inputs resident in HBM, L2 flushed between steps.
+
+Prints ONE JSON line.  value = GFLOP/s of the whole job (banded-LU flops counted
+from the pivots the kernels chose, summed over ranks, divided by the max-over-
+ranks time).  N > 1 runs independent replicas (the single-matrix path has no
+data-parallel split), one per GPU.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "dispatch_lu time & GFLOP/s per matrix; detection HBM GB/s vs peak; speedup over dense"
+WORKLOAD = "n4096_kl16_ku16"
+FP64_PEAK_GFLOPS = 1250.0  # nominal dense FP64 of one GB300 (152 SMs x 2 DFMA/clk x 2 flop x ~2.07 GHz)
+FALLBACK_HBM_GBS = 6800.0
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured (MEASURED_PEAKS.json, copy bandwidth)"
+    return FALLBACK_HBM_GBS, "fallback 6.8 TB/s (no MEASURED_PEAKS.json)"
+
+
+def band_flops(ipiv: np.ndarray, diag: np.ndarray, n: int, kl: int, ku: int) -> int:
+    """sum_j [1 + km + 2*km*(ju_j - j)] over columns with a nonzero pivot, where
+    ju_j is the running reach of U: max over k <= j of min(k + ku + p_k, n-1)."""
+    j = np.arange(n, dtype=np.int64)
+    p = ipiv.astype(np.int64) - 1 - j
+    nzp = diag != 0.0
+    reach = np.where(nzp, np.minimum(j + ku + p, n - 1), 0)
+    ju = np.maximum.accumulate(reach)
+    km = np.minimum(kl, n - 1 - j)
+    per = 1 + km + 2 * km * (ju - j)
+    return int(np.sum(np.where(nzp, per, 0)))
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle reasons sampled every 100 ms in the background."""
+
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.tmp = tempfile.NamedTemporaryFile(prefix="clocks_", suffix=".csv", delete=False)
+        self.tmp.close()
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100", "-i", str(self.index)],
+                                         stdout=open(self.tmp.name, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float):
+        rows = []
+        try:
+            with open(self.tmp.name) as f:
+                for line in f:
+                    parts = [x.strip() for x in line.split(",")]
+                    if len(parts) < 10:
+                        continue
+                    try:
+                        ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                        rows.append((ts, float(parts[2]), float(parts[3]), parts[6:10]))
+                    except ValueError:
+                        continue
+        finally:
+            os.unlink(self.tmp.name)
+        inside = [r for r in rows if t0 - 1.0 <= r[0] <= t1 + 1.0] or rows
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in inside for k in range(4) if r[3][k].lower() == "active"})
+        return {"sm_mhz": statistics.median(r[1] for r in inside), "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": reasons, "samples": len(inside)}
+
+
+def cpu_oracle_dispatch(A_np: np.ndarray, ldab: int, budget_s: float, max_steps: int):
+    """Time the CPU oracle's dispatch (detect + decide + convert + banded LU) on the
+    whole matrix, repeated while the time budget lasts."""
+    import oracle
+    oracle.build()
+    times, res = [], None
+    t_start = time.perf_counter()
+    while len(times) < max_steps:
+        t0 = time.perf_counter()
+        res = oracle.dispatch_lu(A_np, ldab)
+        times.append(time.perf_counter() - t0)
+        if time.perf_counter() - t_start > budget_s:
+            break
+    return times, res
+
+
+def run_reference(args):
+    """The oracle, as it stands, on this host's cores: one step = one dispatch of the workload."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2608_22099_gb300.workloads import WORKLOADS, make_workload
+    w = WORKLOADS[WORKLOAD]
+    A = make_workload(w).numpy()
+    ldab = w.ldab
+    # warm-up steps, then timed steps, all capped so the run ends within a few minutes
+    _, res0 = cpu_oracle_dispatch(A, ldab, budget_s=30.0, max_steps=max(1, args.warmup))
+    times, res = cpu_oracle_dispatch(A, ldab, budget_s=120.0, max_steps=args.steps)
+    flops = band_flops(res["ipiv"], res["AB"][:, w.kl + w.ku], w.n, w.kl, w.ku)
+    t = statistics.mean(times)
+    value = flops / t / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "GFLOP/s", "n_gpus": args.gpus,
+        "steps": len(times), "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "n": w.n, "kl": w.kl, "ku": w.ku, "ldab": ldab},
+        "cpu_baseline": {"value": value, "unit": "GFLOP/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{len(times)} of {args.steps} requested full dispatches of the n={w.n} matrix "
+                                   f"(single-threaded C oracle; time-capped)"},
+        "e2e": {"value": value, "unit": "GFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_22099_gb300 import bandlu
+    from paper_2608_22099_gb300.workloads import WORKLOADS, make_workload
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    w = WORKLOADS[WORKLOAD]
+    n, kl, ku, ldab = w.n, w.kl, w.ku, w.ldab
+    bandlu.load()
+    A = make_workload(w, device=dev)
+    AB = torch.zeros((n, ldab), dtype=torch.float64, device=dev)
+    ipiv = torch.zeros(n, dtype=torch.int32, device=dev)
+    info = torch.zeros(1, dtype=torch.int32, device=dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)  # 512 MiB > L2 (126 MiB)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        rc, gkl, gku = bandlu.dispatch_lu(A, n, n, AB, ldab, ipiv, info, stream)
+        if rc != 0 or (gkl, gku) != (kl, ku):
+            raise RuntimeError(f"dispatch_lu returned {rc} ({gkl}, {gku})")
+
+    for _ in range(max(args.warmup, 3)):
+        flush.fill_(1)
+        step()
+    torch.cuda.synchronize()
+    if int(info.item()) != 0:
+        raise RuntimeError("unexpected zero pivot")
+    flops = band_flops(ipiv.cpu().numpy(), AB[:, kl + ku].cpu().numpy(), n, kl, ku)
+
+    sampler = ClockSampler(local)
+    if rank == 0:
+        sampler.start()
+        time.sleep(0.3)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    for k in range(args.steps):
+        flush.fill_(k)                 # L2 flush between steps, outside the timed events
+        starts[k].record(stream)
+        step()
+        ends[k].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    t_wall1 = time.time()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_ms = torch.tensor([sum(step_ms)], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(total_ms, op=dist.ReduceOp.MAX)
+    ms_per_step = float(total_ms.item()) / args.steps
+    value = world * flops / (ms_per_step * 1e-3) / 1e9
+
+    # stage breakdown through the same C ABI, CUDA events on the launching stream
+    klku = torch.zeros(2, dtype=torch.int32, device=dev)
+    AB2 = torch.zeros_like(AB)
+    ipiv2 = torch.zeros_like(ipiv)
+    info2 = torch.zeros_like(info)
+    reps = min(args.steps, 50)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(reps)]
+    for r in range(reps):
+        flush.fill_(r)
+        e = ev[r]
+        e[0].record(stream)
+        bandlu.check(bandlu.detect_bandwidth(A, n, n, klku, klku.data_ptr() + 4, stream), "detect_bandwidth")
+        e[1].record(stream)
+        bandlu.check(bandlu.dense_to_band(A, n, n, kl, ku, AB2, ldab, stream), "dense_to_band")
+        e[2].record(stream)
+        bandlu.check(bandlu.gbtrf(n, kl, ku, AB2, ldab, ipiv2, info2, stream), "gbtrf")
+        e[3].record(stream)
+    torch.cuda.synchronize()
+    t_detect = statistics.mean(e[0].elapsed_time(e[1]) for e in ev) * 1e-3
+    t_convert = statistics.mean(e[1].elapsed_time(e[2]) for e in ev) * 1e-3
+    t_gbtrf = statistics.mean(e[2].elapsed_time(e[3]) for e in ev) * 1e-3
+    if not (torch.equal(AB2, AB) and torch.equal(ipiv2, ipiv)):
+        raise RuntimeError("stage-by-stage results differ from dispatch_lu")
+
+    hbm_peak, hbm_src = load_peaks()
+    detect_bytes = 8.0 * n * n
+    nnz_band = n * (kl + ku + 1) - kl * (kl + 1) // 2 - ku * (ku + 1) // 2
+    convert_bytes = 8.0 * nnz_band + 8.0 * ldab * n
+    stages = {
+        "detect_us": t_detect * 1e6, "detect_gbs": detect_bytes / t_detect / 1e9,
+        "detect_frac_hbm": detect_bytes / t_detect / 1e9 / hbm_peak,
+        "convert_us": t_convert * 1e6, "convert_gbs": convert_bytes / t_convert / 1e9,
+        "gbtrf_us": t_gbtrf * 1e6, "gbtrf_gflops": flops / t_gbtrf / 1e9,
+        "gbtrf_ns_per_column": t_gbtrf / n * 1e9,
+    }
+    kernels = {"detect": t_detect, "convert": t_convert, "gbtrf": t_gbtrf}
+    dominant = max(kernels, key=kernels.get)
+    if dominant == "gbtrf":
+        achieved = flops / t_gbtrf / 1e9
+        roofline = {"bound": "alu", "achieved": achieved / 1e3, "peak": FP64_PEAK_GFLOPS / 1e3, "unit": "TFLOP/s",
+                    "frac": achieved / FP64_PEAK_GFLOPS, "traffic": None, "kernel": "k_gbtrf_window",
+                    "peak_source": "nominal FP64 (152 SMs x 2 DFMA/clk x 2 flop x 2.07 GHz)",
+                    "note": "one matrix is one serial pivot chain on one SM: latency-bound, see ns_per_column"}
+    elif dominant == "detect":
+        roofline = {"bound": "hbm", "achieved": detect_bytes / t_detect / 1e9, "peak": hbm_peak, "unit": "GB/s",
+                    "frac": detect_bytes / t_detect / 1e9 / hbm_peak, "traffic": None, "kernel": "k_detect_vec",
+                    "peak_source": hbm_src}
+    else:
+        roofline = {"bound": "hbm", "achieved": convert_bytes / t_convert / 1e9, "peak": hbm_peak, "unit": "GB/s",
+                    "frac": convert_bytes / t_convert / 1e9 / hbm_peak, "traffic": None,
+                    "kernel": "k_dense_to_band_tiled", "peak_source": hbm_src}
+
+    # end to end: pinned host input -> device, dispatch_lu, factors back to pinned host memory
+    A_host = A.cpu().pin_memory()
+    AB_host = torch.empty(AB.shape, dtype=AB.dtype).pin_memory()
+    ipiv_host = torch.empty(ipiv.shape, dtype=ipiv.dtype).pin_memory()
+    info_host = torch.empty(info.shape, dtype=info.dtype).pin_memory()
+    A_e2e = torch.empty_like(A)
+    e2e_reps = min(args.steps, 50)
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(e2e_reps)]
+    for r in range(e2e_reps):
+        flush.fill_(r)
+        e0, e1 = e2e_ev[r]
+        e0.record(stream)
+        A_e2e.copy_(A_host, non_blocking=True)
+        rc, _, _ = bandlu.dispatch_lu(A_e2e, n, n, AB, ldab, ipiv, info, stream)
+        bandlu.check(rc, "dispatch_lu")
+        AB_host.copy_(AB, non_blocking=True)
+        ipiv_host.copy_(ipiv, non_blocking=True)
+        info_host.copy_(info, non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
+    e2e_t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(e2e_t, op=dist.ReduceOp.MAX)
+    e2e_value = world * flops / (float(e2e_t.item()) * 1e-3) / 1e9
+    h2d = A_host.numel() * 8
+    d2h = AB_host.numel() * 8 + ipiv_host.numel() * 4 + info_host.numel() * 4
+
+    # the generic algorithm F(N) of Sec. III-A on the same matrix: dense LU (cuSOLVER via torch)
+    dense_ms = []
+    for _ in range(3):
+        Ac = A.clone()
+        torch.cuda.synchronize()
+        a0 = torch.cuda.Event(enable_timing=True); a1 = torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        torch.linalg.lu_factor(Ac)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        dense_ms.append(a0.elapsed_time(a1))
+        del Ac
+    dense_t = statistics.median(dense_ms)
+
+    clocks = None
+    if rank == 0:
+        sampler.stop()
+        clocks = sampler.summary(t_wall0, t_wall1)
+
+    cpu_baseline = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        times, res = cpu_oracle_dispatch(A.cpu().numpy(), ldab, budget_s=20.0, max_steps=1000)
+        cflops = band_flops(res["ipiv"], res["AB"][:, kl + ku], n, kl, ku)
+        cpu_baseline = {"value": cflops / statistics.mean(times) / 1e9, "unit": "GFLOP/s", "cores": 1,
+                        "kind": "oracle",
+                        "sample": f"{len(times)} full dispatches of the n={n} matrix, single-threaded C oracle"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "GFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "n": n, "kl": kl, "ku": ku, "ldab": ldab, "dist": "uniform[-1,1]",
+                       "l2": "flushed between steps (512 MiB write)",
+                       "parallelism": "replicas" if world > 1 else "single"},
+            "dispatch_ms": ms_per_step, "speedup_over_dense": dense_t / ms_per_step, "dense_lu_ms": dense_t,
+            "flops_per_step": flops, "stages": stages, "roofline": roofline,
+            "cpu_baseline": cpu_baseline,
+            "e2e": {"value": e2e_value, "unit": "GFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "ms_per_step": float(e2e_t.item())},
+            "gpu_launches": 3 * args.steps,
+            "clocks": clocks,
+            "wall_s_timed": t_wall1 - t_wall0,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

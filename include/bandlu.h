@@ -1,0 +1,148 @@
+/*
+ * bandlu.h -- C ABI of the GB300 (sm_103a) structure-aware banded LU library.
+ *
+ * The library implements the hot path of the structure-aware dispatch of
+ * Lujan & Edelman, "When Structure is Silent: Opportunities for Algorithmic
+ * Dispatch in Linear Algebra" (HPEC 2025), Sec. II-A (three steps: identify the
+ * structure, convert the format, run the specialised algorithm) instantiated
+ * for LU of banded matrices stored dense (Sec. III, Listing 2).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Dense input A: fp64, ROW-major, n x n, leading dimension lda >= max(1, n):
+ *    element (i, j) is A[i*lda + j].  A is never modified.
+ *  - Band storage AB: fp64, COLUMN-major, ldab x n, LAPACK xGBTRF layout
+ *    (Sec. I-A cites xGBTRF): with kv = kl + ku, element (i, j) of the band
+ *    lives at AB[(kv + i - j) + j*ldab]; rows 0..kl-1 are fill rows that row
+ *    interchanges spill into; ldab >= 2*kl + ku + 1.
+ *  - ipiv: int32, 1-based (LAPACK): row j was interchanged with row ipiv[j]-1.
+ *  - All pointers are DEVICE pointers owned by the caller unless the name starts
+ *    with h_ (host pointer).  Device buffers must not overlap.  The library
+ *    keeps no pointer after a call returns.
+ *  - Work is enqueued on `stream` (0 = legacy default stream) and runs
+ *    asynchronously unless a function says otherwise.
+ *  - Return value: BANDLU_OK, a negative number -i when argument i (1-based) is
+ *    invalid (nothing is enqueued), or one of the positive codes below.  No
+ *    entry point traps, asserts or hangs on the device.
+ *  - Indexing is 64-bit throughout; n is limited to 2^31 - 1 and kl, ku to
+ *    n - 1 (they are int32 in the outputs).
+ */
+#ifndef BANDLU_H
+#define BANDLU_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BANDLU_OK 0
+/* dispatch_lu / dispatch_lu_batched: the dispatch predicate declined the band
+ * path; nothing was factored (AB and ipiv untouched for that matrix). */
+#define BANDLU_NOT_BANDED 1
+/* a CUDA runtime call or kernel launch failed (cudaGetLastError is left set) */
+#define BANDLU_ERR_CUDA 1000
+/* a bounded device-side wait gave up; the results of the call are invalid */
+#define BANDLU_ERR_TIMEOUT 1001
+
+/*
+ * detect_bandwidth -- structure identification, step 1 of Sec. II-A; cost
+ * I(N) ~ O(N^2) (Sec. III-A, Eq. IC-N2); banded_structure(A) in Listing 2.
+ *
+ * Inspects every element of A once and writes
+ *   *d_kl = max(0, max{ i - j : A(i,j) != 0 }),  *d_ku = max(0, max{ j - i : A(i,j) != 0 })
+ * to DEVICE memory.  "Nonzero" is the IEEE comparison a != 0.0: -0.0 counts as
+ * zero; NaN, +-Inf and subnormal values count as nonzero.  An all-zero matrix
+ * or n <= 1 gives (0, 0).  Columns lda-n..lda-1 (padding) are not read as part
+ * of the matrix.
+ * Arguments: 1 A, 2 n >= 0, 3 lda >= max(1,n), 4 d_kl (non-null), 5 d_ku (non-null).
+ * Scratch: none.  Fastest when A is 16-byte aligned and lda is even.
+ */
+int detect_bandwidth(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t stream);
+
+/*
+ * dense_to_band -- format conversion, step 2 of Sec. II-A; cost C(N)
+ * (Sec. III-A, Eq. IC-N2); BandedMatrix(A) in Listing 2.
+ *
+ * Writes all ldab x n entries of AB: AB(kv+i-j, j) = A(i,j) for
+ * max(0, j-ku) <= i <= min(n-1, j+kl), and +0.0 everywhere else (fill rows,
+ * the corner triangles and any rows beyond 2*kl+ku).  Entries of A outside the
+ * band are not read.
+ * Arguments: 1 A, 2 lda >= max(1,n), 3 n >= 0, 4 kl >= 0, 5 ku >= 0, 6 AB,
+ * 7 ldab >= 2*kl+ku+1.  kl and ku must be less than n when n > 0.
+ */
+int dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                  cudaStream_t stream);
+
+/*
+ * gbtrf -- banded LU with partial pivoting, step 3 of Sec. II-A; cost
+ * f(N) ~ O(N*P*Q) (Sec. III-A, Eq. S-N-N3); DGBTRF in Listing 2.
+ *
+ * Factors the band in AB in place as A = P_0 L_0 P_1 L_1 ... P_{n-1} L_{n-1} U
+ * with LAPACK xGBTRF semantics: the pivot of column j is the FIRST entry of
+ * largest magnitude among rows j..min(n-1, j+kl); the interchange is applied to
+ * the columns of U; the multipliers l = a * (1/pivot) (a reciprocal, then one
+ * multiply) of column j are stored in AB rows kv+1..kv+kl of column j, not
+ * permuted by later interchanges; the trailing update is a = fma(-l, u, a) and
+ * is skipped for a column whose pivot-row entry u is exactly zero.  U occupies
+ * rows 0..kv.  The fill rows 0..kl-1 need not be zero on entry.
+ * On exit *d_info (DEVICE) is 0, or j+1 for the first column j whose pivot is
+ * exactly zero (that column is left unscaled and elimination continues, as
+ * LAPACK does; this is not an error return).
+ * Arguments: 1 n >= 0, 2 kl >= 0, 3 ku >= 0, 4 AB, 5 ldab >= 2*kl+ku+1,
+ * 6 ipiv (n int32, device), 7 d_info (device).
+ * Scratch: none.  NaN entries in a pivot column give unspecified pivots.
+ */
+int gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t stream);
+
+/*
+ * dispatch_lu -- the whole strategy of Sec. II-A for one matrix
+ * (structure_aware_lu of Listing 2 without the dense branch).
+ *
+ * Runs detect_bandwidth, reads (kl, ku) back to the host (the call waits for
+ * `stream` once), applies the dispatch predicate, and if it holds runs
+ * dense_to_band and gbtrf on `stream` (those two stay asynchronous).
+ * The predicate is the speedup constraint of Eq. su-con (Sec. II-B),
+ * I(N) + C(N) + f(N) < F(N), with the operation counts I = n^2,
+ * C = n*(kl+ku+1), f = n*kl*(2*(kl+ku)+1) (worst-case fill) and F = 2n^3/3,
+ * evaluated exactly in integers, together with the capacity check
+ * 2*kl+ku+1 <= ldab.
+ * Returns BANDLU_OK (band path enqueued; *d_info is written by gbtrf) or
+ * BANDLU_NOT_BANDED (nothing further enqueued; AB, ipiv, d_info untouched).
+ * *h_kl and *h_ku (HOST) receive the detected bandwidths in both cases.
+ * Arguments: 1 A, 2 n, 3 lda, 4 AB, 5 ldab >= 1, 6 ipiv, 7 h_kl, 8 h_ku, 9 d_info.
+ * Scratch: 8 bytes of device memory for the detected bandwidths, taken from the
+ * stream-ordered allocator (cudaMallocAsync) and released before returning.
+ */
+int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *h_kl,
+                int *h_ku, int *d_info, cudaStream_t stream);
+
+/*
+ * dispatch_lu_batched -- the strategy of Sec. II-A applied to `batch`
+ * independent n x n matrices in one call, with no host round trip.
+ *
+ * Matrix b is read from A + b*strideA (leading dimension lda); its band goes to
+ * AB + b*strideAB (leading dimension ldab), its pivots to ipiv + b*strideP.
+ * Every matrix gets its own (kl, ku) and its own predicate decision (as in
+ * dispatch_lu, with the shared capacity ldab); per-matrix results go to the
+ * DEVICE arrays d_kl[b], d_ku[b], d_info[b] and d_status[b] (BANDLU_OK or
+ * BANDLU_NOT_BANDED; a declined matrix's AB and ipiv are untouched and its
+ * d_info is 0).
+ * Arguments: 1 A, 2 n, 3 lda, 4 strideA >= n*lda, 5 batch >= 0, 6 AB,
+ * 7 ldab >= 1, 8 strideAB >= n*ldab, 9 ipiv, 10 strideP >= n, 11 d_kl, 12 d_ku,
+ * 13 d_info, 14 d_status.
+ * Scratch: none.
+ */
+int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,
+                        int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku,
+                        int *d_info, int *d_status, cudaStream_t stream);
+
+/* Version string of the library build (host, static storage). */
+const char *bandlu_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BANDLU_H */

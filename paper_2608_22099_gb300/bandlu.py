@@ -1,0 +1,117 @@
+"""Thin ctypes binding of the C ABI in include/bandlu.h (argument marshalling only).
+
+Every function has the C name and the C argument order.  Pointer arguments take
+a torch tensor (its data_ptr is passed) or a raw integer address; ``stream``
+takes a torch.cuda.Stream, a raw cudaStream_t integer, or None for torch's
+current stream.  All arithmetic runs in the CUDA library; there is no CPU or
+PyTorch fallback: if the library is missing or fails to load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from . import build as _build
+
+BANDLU_OK = 0
+BANDLU_NOT_BANDED = 1
+BANDLU_ERR_CUDA = 1000
+BANDLU_ERR_TIMEOUT = 1001
+
+_lock = threading.Lock()
+_lib = None
+
+
+class BandLUError(RuntimeError):
+    pass
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load():
+    """Load libbandlu.so (building it first if the sources are newer)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if not _build.up_to_date():
+            try:
+                path = _build.build()
+            except Exception as e:  # noqa: BLE001 - re-raised with context
+                raise BandLUError(f"the CUDA library could not be built: {e}") from e
+        if not os.path.exists(path):
+            raise BandLUError(f"CUDA library missing at {path}")
+        lib = ctypes.CDLL(path)
+        vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+        lib.detect_bandwidth.argtypes = [vp, i64, i64, vp, vp, vp]
+        lib.dense_to_band.argtypes = [vp, i64, i64, i32, i32, vp, i64, vp]
+        lib.gbtrf.argtypes = [i64, i32, i32, vp, i64, vp, vp, vp]
+        lib.dispatch_lu.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
+        lib.dispatch_lu_batched.argtypes = [vp, i64, i64, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
+        for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "dispatch_lu", "dispatch_lu_batched"):
+            getattr(lib, f).restype = ctypes.c_int
+        lib.bandlu_version.restype = ctypes.c_char_p
+        lib.bandlu_version.argtypes = []
+        _lib = lib
+        return lib
+
+
+def _ptr(x) -> int:
+    if x is None:
+        return 0
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def _stream(s) -> int:
+    if s is None:
+        import torch
+        return int(torch.cuda.current_stream().cuda_stream)
+    if isinstance(s, int):
+        return s
+    return int(s.cuda_stream)
+
+
+def version() -> str:
+    return load().bandlu_version().decode()
+
+
+def detect_bandwidth(A, n: int, lda: int, d_kl, d_ku, stream=None) -> int:
+    return load().detect_bandwidth(_ptr(A), n, lda, _ptr(d_kl), _ptr(d_ku), _stream(stream))
+
+
+def dense_to_band(A, lda: int, n: int, kl: int, ku: int, AB, ldab: int, stream=None) -> int:
+    return load().dense_to_band(_ptr(A), lda, n, kl, ku, _ptr(AB), ldab, _stream(stream))
+
+
+def gbtrf(n: int, kl: int, ku: int, AB, ldab: int, ipiv, d_info, stream=None) -> int:
+    return load().gbtrf(n, kl, ku, _ptr(AB), ldab, _ptr(ipiv), _ptr(d_info), _stream(stream))
+
+
+def dispatch_lu(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -> tuple[int, int, int]:
+    """Returns (status, kl, ku); kl and ku are the host outputs of the C call."""
+    kl, ku = ctypes.c_int(-1), ctypes.c_int(-1)
+    rc = load().dispatch_lu(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), ctypes.addressof(kl),
+                            ctypes.addressof(ku), _ptr(d_info), _stream(stream))
+    return rc, kl.value, ku.value
+
+
+def dispatch_lu_batched(A, n: int, lda: int, strideA: int, batch: int, AB, ldab: int, strideAB: int, ipiv,
+                        strideP: int, d_kl, d_ku, d_info, d_status, stream=None) -> int:
+    return load().dispatch_lu_batched(_ptr(A), n, lda, strideA, batch, _ptr(AB), ldab, strideAB, _ptr(ipiv),
+                                      strideP, _ptr(d_kl), _ptr(d_ku), _ptr(d_info), _ptr(d_status),
+                                      _stream(stream))
+
+
+def check(rc: int, what: str = "call") -> int:
+    """Raise BandLUError for an error status (negative or >= BANDLU_ERR_CUDA)."""
+    if rc < 0:
+        raise BandLUError(f"{what}: invalid argument {-rc}")
+    if rc >= BANDLU_ERR_CUDA:
+        raise BandLUError(f"{what}: status {rc}")
+    return rc

@@ -1,0 +1,103 @@
+// api.cu -- the C ABI (declared in include/bandlu.h): argument checks, then the
+// launches of detect.cu, convert.cu, gbtrf.cu and batched.cu.
+#include <climits>
+
+#include "common.cuh"
+
+namespace {
+
+inline bool bad_n(int64_t n) { return n < 0 || n > (int64_t)INT_MAX; }
+inline int64_t max1(int64_t n) { return n > 1 ? n : 1; }
+
+}  // namespace
+
+extern "C" {
+
+const char *bandlu_version(void) { return "bandlu 0.1 (sm_103a)"; }
+
+int detect_bandwidth(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t stream) {
+  if (bad_n(n)) return -2;
+  if (A == nullptr && n > 0) return -1;
+  if (lda < max1(n)) return -3;
+  if (d_kl == nullptr) return -4;
+  if (d_ku == nullptr) return -5;
+  return bandlu::launch_detect(A, n, lda, d_kl, d_ku, stream);
+}
+
+int dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                  cudaStream_t stream) {
+  if (bad_n(n)) return -3;
+  if (A == nullptr && n > 0) return -1;
+  if (lda < max1(n)) return -2;
+  if (kl < 0) return -4;
+  if (ku < 0) return -5;
+  if (AB == nullptr && n > 0) return -6;
+  if (ldab < 2 * (int64_t)kl + ku + 1) return -7;
+  return bandlu::launch_dense_to_band(A, lda, n, kl, ku, AB, ldab, stream);
+}
+
+int gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t stream) {
+  if (bad_n(n)) return -1;
+  if (kl < 0) return -2;
+  if (ku < 0) return -3;
+  if (AB == nullptr && n > 0) return -4;
+  if (ldab < 2 * (int64_t)kl + ku + 1) return -5;
+  if (ipiv == nullptr && n > 0) return -6;
+  if (d_info == nullptr) return -7;
+  return bandlu::launch_gbtrf(n, kl, ku, AB, ldab, ipiv, d_info, stream);
+}
+
+int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *h_kl, int *h_ku,
+                int *d_info, cudaStream_t stream) {
+  if (A == nullptr && n > 0) return -1;
+  if (bad_n(n)) return -2;
+  if (lda < max1(n)) return -3;
+  if (AB == nullptr && n > 0) return -4;
+  if (ldab < 1) return -5;
+  if (ipiv == nullptr && n > 0) return -6;
+  if (h_kl == nullptr) return -7;
+  if (h_ku == nullptr) return -8;
+  if (d_info == nullptr) return -9;
+  int *d_klku = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&d_klku), 2 * sizeof(int), stream) != cudaSuccess)
+    return BANDLU_ERR_CUDA;
+  int rc = bandlu::launch_detect(A, n, lda, d_klku, d_klku + 1, stream);
+  int h[2] = {0, 0};
+  if (rc == BANDLU_OK && cudaMemcpyAsync(h, d_klku, sizeof(h), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    rc = BANDLU_ERR_CUDA;
+  if (cudaFreeAsync(d_klku, stream) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (cudaStreamSynchronize(stream) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (rc != BANDLU_OK) return rc;
+  *h_kl = h[0];
+  *h_ku = h[1];
+  if (!bandlu::predicate_banded(n, h[0], h[1], ldab)) return BANDLU_NOT_BANDED;
+  rc = bandlu::launch_dense_to_band(A, lda, n, h[0], h[1], AB, ldab, stream);
+  if (rc != BANDLU_OK) return rc;
+  return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream);
+}
+
+int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,
+                        int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku,
+                        int *d_info, int *d_status, cudaStream_t stream) {
+  const bool work = n > 0 && batch > 0;
+  if (A == nullptr && work) return -1;
+  if (bad_n(n)) return -2;
+  if (lda < max1(n)) return -3;
+  if (strideA < n * lda) return -4;
+  if (batch < 0) return -5;
+  if (AB == nullptr && work) return -6;
+  if (ldab < 1) return -7;
+  if (strideAB < n * ldab) return -8;
+  if (ipiv == nullptr && work) return -9;
+  if (strideP < n) return -10;
+  if ((d_kl == nullptr || d_ku == nullptr || d_info == nullptr || d_status == nullptr) && batch > 0) {
+    if (d_kl == nullptr) return -11;
+    if (d_ku == nullptr) return -12;
+    if (d_info == nullptr) return -13;
+    return -14;
+  }
+  return bandlu::launch_batched(A, n, lda, strideA, batch, AB, ldab, strideAB, ipiv, strideP, d_kl, d_ku, d_info,
+                                d_status, stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,238 @@
+// batched.cu -- the strategy of Sec. II-A over a batch of independent matrices,
+// with no host round trip: every matrix gets its own identification, decision,
+// conversion and factorisation.
+//
+//  * k_batch_scan_convert: one block per matrix.  Warps stride over rows and
+//    lanes over 16-byte vectors of a row (consecutive addresses); the block
+//    folds the largest i-j / j-i over nonzeros, applies the dispatch predicate
+//    and, for a banded matrix, writes its band storage (reading the band back
+//    from the matrix it has just scanned, which is still in L2).
+//  * k_batch_factor: one warp per matrix.  The matrix's band is staged into
+//    shared memory when it fits, factored there with the unblocked
+//    elimination (same order of operations as the single-matrix kernels), and
+//    written back.
+#include <climits>
+
+#include "common.cuh"
+
+namespace bandlu {
+namespace {
+
+__global__ void __launch_bounds__(256) k_batch_scan_convert(const double *__restrict__ A, long long n, long long lda,
+                                                            long long strideA, long long batch, double *__restrict__ AB,
+                                                            long long ldab, long long strideAB, int *__restrict__ d_kl,
+                                                            int *__restrict__ d_ku, int *__restrict__ d_info,
+                                                            int *__restrict__ d_status, int vec) {
+  __shared__ int s_l[8], s_u[8];
+  __shared__ int s_kl, s_ku, s_banded;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (long long b = blockIdx.x; b < batch; b += gridDim.x) {
+    const double *Ab = A + b * strideA;
+    int lmax = 0, umax = 0;
+    if (vec) {
+      const long long nv = (n + 1) / 2;
+      for (long long i = warp; i < n; i += nw) {
+        const ulonglong2 *row = reinterpret_cast<const ulonglong2 *>(Ab + i * lda);
+        for (long long v0 = lane; v0 < nv; v0 += 32 * 4) {
+          ulonglong2 x[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const long long v = v0 + 32 * u;
+            x[u] = v < nv ? __ldcs(row + v) : make_ulonglong2(0ull, 0ull);
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if (((x[u].x << 1) | (x[u].y << 1)) != 0ull) {
+              const long long j0 = 2 * (v0 + 32 * u);
+              if (nz_bits(x[u].x)) {
+                lmax = max(lmax, (int)(i - j0));
+                umax = max(umax, (int)(j0 - i));
+              }
+              if (nz_bits(x[u].y) && j0 + 1 < n) {
+                lmax = max(lmax, (int)(i - j0 - 1));
+                umax = max(umax, (int)(j0 + 1 - i));
+              }
+            }
+          }
+        }
+      }
+    } else {
+      for (long long i = warp; i < n; i += nw) {
+        const unsigned long long *row = reinterpret_cast<const unsigned long long *>(Ab + i * lda);
+        for (long long j = lane; j < n; j += 32) {
+          if (nz_bits(__ldcs(row + j))) {
+            lmax = max(lmax, (int)(i - j));
+            umax = max(umax, (int)(j - i));
+          }
+        }
+      }
+    }
+    lmax = __reduce_max_sync(FULL, lmax);
+    umax = __reduce_max_sync(FULL, umax);
+    if (lane == 0) {
+      s_l[warp] = lmax;
+      s_u[warp] = umax;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int kl = 0, ku = 0;
+      for (int w = 0; w < nw; ++w) {
+        kl = max(kl, s_l[w]);
+        ku = max(ku, s_u[w]);
+      }
+      const bool banded = predicate_banded(n, kl, ku, ldab);
+      s_kl = kl;
+      s_ku = ku;
+      s_banded = banded ? 1 : 0;
+      d_kl[b] = kl;
+      d_ku[b] = ku;
+      d_info[b] = 0;
+      d_status[b] = banded ? BANDLU_OK : BANDLU_NOT_BANDED;
+    }
+    __syncthreads();
+    if (s_banded) {
+      const long long kl = s_kl, ku = s_ku, kv = kl + ku;
+      double *ABb = AB + b * strideAB;
+      const long long total = n * ldab;
+      for (long long e = threadIdx.x; e < total; e += blockDim.x) {
+        const long long j = e / ldab;
+        const long long r = e - j * ldab;
+        const long long i = j - kv + r;
+        double v = 0.0;
+        if (r >= kl && r <= kv + kl && i >= 0 && i < n) v = Ab[i * lda + j];
+        ABb[e] = v;
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// Unblocked banded elimination by one warp on band storage `ab` (shared or
+// global memory).  Returns info.
+__device__ int warp_gbtrf(double *ab, long long ldab, long long n, int kl, int ku, int *ipiv) {
+  const int lane = threadIdx.x & 31;
+  const long long kv = (long long)kl + ku;
+  if (kl > 0) {
+    for (long long e = lane; e < n * kl; e += 32) {
+      const long long c = e / kl, r = e - c * kl;
+      ab[r + c * ldab] = 0.0;
+    }
+  }
+  __syncwarp();
+  long long ju = 0;
+  int info = 0;
+  for (long long j = 0; j < n; ++j) {
+    const long long km = min((long long)kl, n - 1 - j);
+    double *col = ab + j * ldab;
+    KeyIdx best{0ull, LLONG_MAX};
+    for (long long t = lane; t <= km; t += 32) best = better(best, KeyIdx{abs_key(col[kv + t]), t});
+    best = warp_reduce_keyidx(best);
+    const long long p = best.idx;
+    const double pv = col[kv + p];
+    if (lane == 0) ipiv[j] = (int)(j + p + 1);
+    __syncwarp();
+    if (nz(pv)) {
+      ju = max(ju, min(j + ku + p, n - 1));
+      if (p != 0) {
+        for (long long c = j + lane; c <= ju; c += 32) {
+          double *x = ab + (kv + j - c) + c * ldab;
+          double *y = ab + (kv + j + p - c) + c * ldab;
+          const double t0 = *x;
+          *x = *y;
+          *y = t0;
+        }
+        __syncwarp();
+      }
+      if (km > 0) {
+        const double r = 1.0 / pv;
+        for (long long t = 1 + lane; t <= km; t += 32) col[kv + t] *= r;
+        __syncwarp();
+        const long long tot = (ju - j) * km;
+        for (long long e = lane; e < tot; e += 32) {
+          const long long cc = e / km, t = 1 + (e - cc * km);
+          const long long c = j + 1 + cc;
+          double *colc = ab + c * ldab;
+          const double u = colc[kv + j - c];
+          if (nz(u)) colc[kv + j + t - c] = fma(-col[kv + t], u, colc[kv + j + t - c]);
+        }
+        __syncwarp();
+      }
+    } else if (info == 0) {
+      info = (int)(j + 1);
+    }
+  }
+  return info;
+}
+
+__global__ void __launch_bounds__(128) k_batch_factor(long long n, long long batch, double *__restrict__ AB,
+                                                      long long ldab, long long strideAB, int *__restrict__ ipiv,
+                                                      long long strideP, const int *__restrict__ d_kl,
+                                                      const int *__restrict__ d_ku, int *__restrict__ d_info,
+                                                      const int *__restrict__ d_status, int staged) {
+  extern __shared__ double stage[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
+  const long long b = (long long)blockIdx.x * wpb + warp;
+  if (b >= batch) return;  // whole warp leaves together
+  if (d_status[b] != BANDLU_OK) return;
+  const int kl = d_kl[b], ku = d_ku[b];
+  double *ABb = AB + b * strideAB;
+  int info;
+  if (staged) {
+    double *s = stage + (long long)warp * n * ldab;
+    const long long total = n * ldab;
+    for (long long e = lane; e < total; e += 32) s[e] = ABb[e];
+    __syncwarp();
+    info = warp_gbtrf(s, ldab, n, kl, ku, ipiv + b * strideP);
+    __syncwarp();
+    for (long long e = lane; e < total; e += 32) ABb[e] = s[e];
+  } else {
+    info = warp_gbtrf(ABb, ldab, n, kl, ku, ipiv + b * strideP);
+  }
+  if (lane == 0) d_info[b] = info;
+}
+
+int num_sms_b() {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 152;
+  }
+  return sms;
+}
+
+constexpr int kStageMaxBytes = 24 * 1024;
+
+}  // namespace
+
+int launch_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB, int64_t ldab,
+                   int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku, int *d_info, int *d_status,
+                   cudaStream_t s) {
+  if (batch == 0) return BANDLU_OK;
+  const int vec = ((reinterpret_cast<uintptr_t>(A) & 15u) == 0) && (lda % 2 == 0) && (strideA % 2 == 0);
+  long long grid1 = batch;
+  const long long cap = (long long)num_sms_b() * 64;
+  if (grid1 > cap) grid1 = cap;
+  k_batch_scan_convert<<<(unsigned)grid1, 256, 0, s>>>(A, n, lda, strideA, batch, AB, ldab, strideAB, d_kl, d_ku,
+                                                       d_info, d_status, vec);
+  BANDLU_CHECK_LAUNCH();
+  if (n == 0) return BANDLU_OK;
+  const long long per = n * ldab * (long long)sizeof(double);
+  const int wpb = 4;
+  const int staged = per <= kStageMaxBytes ? 1 : 0;
+  const size_t smem = staged ? (size_t)per * wpb : 0;
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(k_batch_factor, cudaFuncAttributeMaxDynamicSharedMemorySize, kStageMaxBytes * wpb) !=
+        cudaSuccess)
+      return BANDLU_ERR_CUDA;
+    attr = true;
+  }
+  const long long grid2 = (batch + wpb - 1) / wpb;
+  k_batch_factor<<<(unsigned)grid2, 32 * wpb, smem, s>>>(n, batch, AB, ldab, strideAB, ipiv, strideP, d_kl, d_ku,
+                                                         d_info, d_status, staged);
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+}  // namespace bandlu

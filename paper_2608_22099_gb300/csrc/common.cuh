@@ -1,0 +1,81 @@
+// common.cuh -- shared device helpers of the banded LU library (sm_103a).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "bandlu.h"
+
+namespace bandlu {
+
+constexpr unsigned FULL = 0xffffffffu;
+
+// IEEE "a != 0.0" on the bit pattern: true for every value except +0.0 and -0.0
+// (NaN, +-Inf and subnormals are nonzero).  Integer-only, so it never issues on
+// the FP64 pipe.
+__device__ __forceinline__ bool nz_bits(unsigned long long b) { return (b << 1) != 0ull; }
+__device__ __forceinline__ bool nz(double x) { return nz_bits((unsigned long long)__double_as_longlong(x)); }
+
+// |x| as an unsigned key: for non-NaN doubles, |x| < |y| iff key(x) < key(y).
+__device__ __forceinline__ unsigned long long abs_key(double x) {
+  return (unsigned long long)__double_as_longlong(x) & 0x7fffffffffffffffull;
+}
+
+// First lane holding the largest key among all 32 lanes (ties -> lowest lane).
+// Exact on 63-bit keys using two 32-bit max reductions and a ballot.
+__device__ __forceinline__ int warp_argmax_first(unsigned long long key) {
+  const unsigned hi = (unsigned)(key >> 32), lo = (unsigned)key;
+  const unsigned mhi = __reduce_max_sync(FULL, hi);
+  const unsigned lo2 = (hi == mhi) ? lo : 0u;
+  const unsigned mlo = __reduce_max_sync(FULL, lo2);
+  const unsigned win = __ballot_sync(FULL, hi == mhi && lo == mlo);
+  return __ffs(win) - 1;
+}
+
+// (key, index) pair that prefers the larger key and, on a tie, the smaller index.
+struct KeyIdx {
+  unsigned long long key;
+  long long idx;
+};
+__device__ __forceinline__ KeyIdx better(KeyIdx a, KeyIdx b) {
+  if (b.key > a.key || (b.key == a.key && b.idx < a.idx)) return b;
+  return a;
+}
+__device__ __forceinline__ KeyIdx warp_reduce_keyidx(KeyIdx v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    KeyIdx o;
+    o.key = __shfl_xor_sync(FULL, v.key, off);
+    o.idx = __shfl_xor_sync(FULL, v.idx, off);
+    v = better(v, o);
+  }
+  return v;
+}
+
+// Dispatch predicate (Eq. su-con with integer operation counts, and the storage
+// capacity): banded iff 3*(n^2 + n*(kl+ku+1) + n*kl*(2*(kl+ku)+1)) < 2*n^3 and
+// 2*kl+ku+1 <= ldab.  128-bit arithmetic: exact for every n < 2^31.
+__host__ __device__ inline bool predicate_banded(long long n, long long kl, long long ku, long long ldab) {
+  if (2 * kl + ku + 1 > ldab) return false;
+  const __int128 N = n, L = kl, U = ku;
+  const __int128 lhs = 3 * (N * N + N * (L + U + 1) + N * L * (2 * (L + U) + 1));
+  return lhs < 2 * N * N * N;
+}
+
+}  // namespace bandlu
+
+#define BANDLU_CHECK_LAUNCH()                         \
+  do {                                                \
+    if (cudaPeekAtLastError() != cudaSuccess) return BANDLU_ERR_CUDA; \
+  } while (0)
+
+// Launchers shared between the C-ABI translation unit and the kernel units.
+namespace bandlu {
+int launch_detect(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t s);
+int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                         cudaStream_t s);
+int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s);
+int launch_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,
+                   int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku, int *d_info,
+                   int *d_status, cudaStream_t s);
+}  // namespace bandlu

@@ -1,0 +1,90 @@
+// convert.cu -- format conversion (Sec. II-A step 2; C(N), Eq. IC-N2).
+//
+// Dense row-major A -> LAPACK band storage AB (column-major, ldab x n).  A block
+// owns T consecutive output columns [j0, j0+T), i.e. the contiguous run
+// AB[j0*ldab, (j0+T)*ldab).  It zeroes a T x ldab shared-memory tile laid out
+// exactly like that run, gathers the band part of rows j0-ku .. j0+T-1+kl of A
+// into it (each row's band segment is contiguous in A, so a warp reads it with
+// consecutive addresses), and streams the tile out with consecutive stores.
+// Only band entries of A are read; every AB entry is written.
+#include "common.cuh"
+
+namespace bandlu {
+namespace {
+
+__global__ void __launch_bounds__(256) k_dense_to_band_tiled(const double *__restrict__ A, long long lda, long long n,
+                                                             int kl, int ku, double *__restrict__ AB, long long ldab,
+                                                             int T) {
+  extern __shared__ double tile[];  // T * ldab, tile[c*ldab + r] = AB(r, j0+c)
+  const long long kv = (long long)kl + ku;
+  const long long j0 = (long long)blockIdx.x * T;
+  const int tcols = (int)min((long long)T, n - j0);
+  const long long tsize = (long long)tcols * ldab;
+  for (long long e = threadIdx.x; e < tsize; e += blockDim.x) tile[e] = 0.0;
+  __syncthreads();
+  const long long i_lo = max(0ll, j0 - ku);
+  const long long i_hi = min(n - 1, j0 + tcols - 1 + kl);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+  for (long long i = i_lo + warp; i <= i_hi; i += nwarps) {
+    const long long c_lo = max(j0, i - kl);
+    const long long c_hi = min(min(j0 + tcols - 1, i + ku), n - 1);
+    for (long long c = c_lo + lane; c <= c_hi; c += 32) {
+      tile[(c - j0) * ldab + (kv + i - c)] = A[i * lda + c];
+    }
+  }
+  __syncthreads();
+  double *out = AB + j0 * ldab;
+  for (long long e = threadIdx.x; e < tsize; e += blockDim.x) out[e] = tile[e];
+}
+
+// Direct form for very tall band storage: one thread per AB entry, consecutive
+// threads on consecutive AB rows (coalesced stores; reads of A are strided).
+__global__ void __launch_bounds__(256) k_dense_to_band_direct(const double *__restrict__ A, long long lda, long long n,
+                                                              int kl, int ku, double *__restrict__ AB, long long ldab) {
+  const long long kv = (long long)kl + ku;
+  const long long total = n * ldab;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long j = e / ldab;
+    const long long r = e - j * ldab;
+    const long long i = j - kv + r;
+    double v = 0.0;
+    if (r >= kl && r <= kv + kl && i >= 0 && i < n) v = A[i * lda + j];
+    AB[e] = v;
+  }
+}
+
+constexpr int kTileSmemMax = 96 * 1024;
+
+}  // namespace
+
+int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                         cudaStream_t s) {
+  if (n == 0) return BANDLU_OK;
+  const long long per_col = ldab * (long long)sizeof(double);
+  if (per_col <= kTileSmemMax) {
+    // T columns per block: enough blocks to cover the SMs for small n, at most 32.
+    int T = (int)min(32ll, (long long)kTileSmemMax / per_col);
+    while (T > 1 && (n + T - 1) / T < 304) T >>= 1;
+    if (T < 1) T = 1;
+    const size_t smem = (size_t)T * per_col;
+    static bool attr_set = false;
+    if (!attr_set) {
+      if (cudaFuncSetAttribute(k_dense_to_band_tiled, cudaFuncAttributeMaxDynamicSharedMemorySize, kTileSmemMax) !=
+          cudaSuccess)
+        return BANDLU_ERR_CUDA;
+      attr_set = true;
+    }
+    const long long blocks = (n + T - 1) / T;
+    k_dense_to_band_tiled<<<(unsigned)blocks, 256, smem, s>>>(A, lda, n, kl, ku, AB, ldab, T);
+  } else {
+    const long long total = n * ldab;
+    long long blocks = (total + 255) / 256;
+    if (blocks > 152ll * 32) blocks = 152ll * 32;
+    k_dense_to_band_direct<<<(unsigned)blocks, 256, 0, s>>>(A, lda, n, kl, ku, AB, ldab);
+  }
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+}  // namespace bandlu

@@ -1,0 +1,149 @@
+// detect.cu -- structure identification (Sec. II-A step 1; I(N) ~ O(N^2), Eq. IC-N2).
+//
+// One HBM-bound pass over the n x n row-major matrix.  Work items are
+// (row, segment) pairs; a segment is blockDim.x * U consecutive 16-byte vectors
+// of one row, so every warp load is a contiguous 512-byte run.  Each thread
+// keeps the largest i-j and j-i over the nonzeros it sees, the block folds them
+// with warp max-reductions, and one thread per block folds the block result
+// into the two outputs with atomicMax.  The nonzero test is integer-only
+// ((bits << 1) != 0), so the FP64 pipe is never used.
+#include "common.cuh"
+
+namespace bandlu {
+namespace {
+
+__device__ __forceinline__ void block_fold(int lmax, int umax, int *d_kl, int *d_ku) {
+  __shared__ int s_l[32], s_u[32];
+  lmax = __reduce_max_sync(FULL, lmax);
+  umax = __reduce_max_sync(FULL, umax);
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) { s_l[w] = lmax; s_u[w] = umax; }
+  __syncthreads();
+  if (w == 0) {
+    const int nw = blockDim.x >> 5;
+    lmax = lane < nw ? s_l[lane] : 0;
+    umax = lane < nw ? s_u[lane] : 0;
+    lmax = __reduce_max_sync(FULL, lmax);
+    umax = __reduce_max_sync(FULL, umax);
+    if (lane == 0) {
+      if (lmax > 0) atomicMax(d_kl, lmax);
+      if (umax > 0) atomicMax(d_ku, umax);
+    }
+  }
+}
+
+// 16-byte path: A 16-byte aligned and lda even, so every row starts aligned.
+// Vector v of row i holds columns 2v and 2v+1 (2v+1 may be the first padding
+// column when n is odd; it is in bounds because lda >= n+1 then, and ignored).
+template <int U>
+__global__ void __launch_bounds__(512) k_detect_vec(const double *__restrict__ A, long long n, long long lda,
+                                                    long long nv, long long nseg, int *d_kl, int *d_ku) {
+  const long long items = n * nseg;
+  const long long seglen = (long long)blockDim.x * U;
+  int lmax = 0, umax = 0;
+  for (long long it = blockIdx.x; it < items; it += gridDim.x) {
+    const long long i = it / nseg;
+    const long long s = it - i * nseg;
+    const ulonglong2 *row = reinterpret_cast<const ulonglong2 *>(A + i * lda);
+    const long long v0 = s * seglen + threadIdx.x;
+    ulonglong2 x[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const long long v = v0 + (long long)u * blockDim.x;
+      x[u] = v < nv ? __ldcs(row + v) : make_ulonglong2(0ull, 0ull);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (((x[u].x << 1) | (x[u].y << 1)) != 0ull) {  // rare in a banded matrix
+        const long long j0 = 2 * (v0 + (long long)u * blockDim.x);
+        if (nz_bits(x[u].x)) {
+          lmax = max(lmax, (int)(i - j0));
+          umax = max(umax, (int)(j0 - i));
+        }
+        if (nz_bits(x[u].y) && j0 + 1 < n) {
+          lmax = max(lmax, (int)(i - j0 - 1));
+          umax = max(umax, (int)(j0 + 1 - i));
+        }
+      }
+    }
+  }
+  block_fold(lmax, umax, d_kl, d_ku);
+}
+
+// 8-byte path for any alignment / odd lda.
+__global__ void __launch_bounds__(256) k_detect_scalar(const double *__restrict__ A, long long n, long long lda,
+                                                       long long nseg, int *d_kl, int *d_ku) {
+  const long long items = n * nseg;
+  int lmax = 0, umax = 0;
+  for (long long it = blockIdx.x; it < items; it += gridDim.x) {
+    const long long i = it / nseg;
+    const long long s = it - i * nseg;
+    const unsigned long long *row = reinterpret_cast<const unsigned long long *>(A + i * lda);
+    const long long j0 = s * (long long)blockDim.x * 4 + threadIdx.x;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const long long j = j0 + (long long)u * blockDim.x;
+      if (j < n && nz_bits(__ldcs(row + j))) {
+        lmax = max(lmax, (int)(i - j));
+        umax = max(umax, (int)(j - i));
+      }
+    }
+  }
+  block_fold(lmax, umax, d_kl, d_ku);
+}
+
+int num_sms() {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 152;
+  }
+  return sms;
+}
+
+}  // namespace
+
+int launch_detect(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t s) {
+  if (d_ku == d_kl + 1) {
+    if (cudaMemsetAsync(d_kl, 0, 2 * sizeof(int), s) != cudaSuccess) return BANDLU_ERR_CUDA;
+  } else {
+    if (cudaMemsetAsync(d_kl, 0, sizeof(int), s) != cudaSuccess) return BANDLU_ERR_CUDA;
+    if (cudaMemsetAsync(d_ku, 0, sizeof(int), s) != cudaSuccess) return BANDLU_ERR_CUDA;
+  }
+  if (n <= 1) return BANDLU_OK;
+  const int sms = num_sms();
+  const bool vec = ((reinterpret_cast<uintptr_t>(A) & 15u) == 0) && (lda % 2 == 0);
+  if (vec) {
+    const long long nv = (n + 1) / 2;
+    if (nv >= 2048) {
+      const int B = 512;
+      const long long nseg = (nv + (long long)B * 4 - 1) / ((long long)B * 4);
+      const long long items = n * nseg;
+      const long long grid = items < (long long)sms * 4 ? items : (long long)sms * 4;
+      k_detect_vec<4><<<(unsigned)grid, B, 0, s>>>(A, n, lda, nv, nseg, d_kl, d_ku);
+    } else if (nv >= 512) {
+      const int B = 128;
+      const long long nseg = (nv + (long long)B * 4 - 1) / ((long long)B * 4);
+      const long long items = n * nseg;
+      const long long grid = items < (long long)sms * 16 ? items : (long long)sms * 16;
+      k_detect_vec<4><<<(unsigned)grid, B, 0, s>>>(A, n, lda, nv, nseg, d_kl, d_ku);
+    } else {
+      const int B = nv >= 128 ? 128 : 32;
+      const long long nseg = (nv + B - 1) / B;
+      const long long items = n * nseg;
+      const long long grid = items < (long long)sms * 16 ? items : (long long)sms * 16;
+      k_detect_vec<1><<<(unsigned)grid, B, 0, s>>>(A, n, lda, nv, nseg, d_kl, d_ku);
+    }
+  } else {
+    const int B = 256;
+    const long long nseg = (n + (long long)B * 4 - 1) / ((long long)B * 4);
+    const long long items = n * nseg;
+    const long long grid = items < (long long)sms * 8 ? items : (long long)sms * 8;
+    k_detect_scalar<<<(unsigned)grid, B, 0, s>>>(A, n, lda, nseg, d_kl, d_ku);
+  }
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+}  // namespace bandlu

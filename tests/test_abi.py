@@ -1,0 +1,111 @@
+"""The C-ABI library builds, loads and exports every entry point include/bandlu.h
+declares; invalid arguments are rejected on the host before anything is
+enqueued (no GPU needed: these calls never reach CUDA)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_22099_gb300 import bandlu
+from paper_2608_22099_gb300 import build as pbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER_DIR = os.path.join(ROOT, "include")
+
+
+def declared_functions():
+    names = []
+    for h in sorted(os.listdir(HEADER_DIR)):
+        if not h.endswith(".h"):
+            continue
+        text = open(os.path.join(HEADER_DIR, h)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"^\s*(?:const\s+)?\w+\s*\*?\s*(\w+)\s*\(", text, flags=re.M):
+            names.append(m.group(1))
+    return names
+
+
+def test_library_builds_and_exports_every_declared_symbol():
+    path = pbuild.build()
+    assert os.path.exists(path)
+    lib = ctypes.CDLL(path)
+    names = declared_functions()
+    assert {"detect_bandwidth", "dense_to_band", "gbtrf", "dispatch_lu", "dispatch_lu_batched"} <= set(names)
+    for name in names:
+        assert hasattr(lib, name), name
+    assert bandlu.version().startswith("bandlu")
+
+
+DEV = 1 << 20  # a non-null placeholder address: never dereferenced by the host checks
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((DEV, -1, 1, DEV, DEV), -2),
+    ((0, 4, 4, DEV, DEV), -1),
+    ((DEV, 4, 3, DEV, DEV), -3),
+    ((DEV, 4, 4, 0, DEV), -4),
+    ((DEV, 4, 4, DEV, 0), -5),
+    ((DEV, 1 << 31, 1 << 31, DEV, DEV), -2),
+])
+def test_detect_bandwidth_argument_checks(args, expect):
+    assert bandlu.detect_bandwidth(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, 1, 1, DEV, 4), -1),
+    ((DEV, 3, 4, 1, 1, DEV, 4), -2),
+    ((DEV, 4, -1, 1, 1, DEV, 4), -3),
+    ((DEV, 4, 4, -1, 1, DEV, 4), -4),
+    ((DEV, 4, 4, 1, -1, DEV, 4), -5),
+    ((DEV, 4, 4, 1, 1, 0, 4), -6),
+    ((DEV, 4, 4, 1, 1, DEV, 3), -7),
+])
+def test_dense_to_band_argument_checks(args, expect):
+    assert bandlu.dense_to_band(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((-1, 1, 1, DEV, 4, DEV, DEV), -1),
+    ((4, -1, 1, DEV, 4, DEV, DEV), -2),
+    ((4, 1, -1, DEV, 4, DEV, DEV), -3),
+    ((4, 1, 1, 0, 4, DEV, DEV), -4),
+    ((4, 2, 1, DEV, 5, DEV, DEV), -5),
+    ((4, 1, 1, DEV, 4, 0, DEV), -6),
+    ((4, 1, 1, DEV, 4, DEV, 0), -7),
+])
+def test_gbtrf_argument_checks(args, expect):
+    assert bandlu.gbtrf(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, DEV, 4, DEV, DEV), -1),
+    ((DEV, -2, 4, DEV, 4, DEV, DEV), -2),
+    ((DEV, 4, 2, DEV, 4, DEV, DEV), -3),
+    ((DEV, 4, 4, 0, 4, DEV, DEV), -4),
+    ((DEV, 4, 4, DEV, 0, DEV, DEV), -5),
+    ((DEV, 4, 4, DEV, 4, 0, DEV), -6),
+    ((DEV, 4, 4, DEV, 4, DEV, 0), -9),
+])
+def test_dispatch_lu_argument_checks(args, expect):
+    rc, _, _ = bandlu.dispatch_lu(*args, stream=0)
+    assert rc == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, 16, 2, DEV, 4, 16, DEV, 4, DEV, DEV, DEV, DEV), -1),
+    ((DEV, 4, 4, 15, 2, DEV, 4, 16, DEV, 4, DEV, DEV, DEV, DEV), -4),
+    ((DEV, 4, 4, 16, -1, DEV, 4, 16, DEV, 4, DEV, DEV, DEV, DEV), -5),
+    ((DEV, 4, 4, 16, 2, DEV, 4, 15, DEV, 4, DEV, DEV, DEV, DEV), -8),
+    ((DEV, 4, 4, 16, 2, DEV, 4, 16, DEV, 3, DEV, DEV, DEV, DEV), -10),
+    ((DEV, 4, 4, 16, 2, DEV, 4, 16, DEV, 4, DEV, DEV, DEV, 0), -14),
+])
+def test_dispatch_lu_batched_argument_checks(args, expect):
+    assert bandlu.dispatch_lu_batched(*args, stream=0) == expect
+
+
+def test_binding_has_the_c_names():
+    for name in declared_functions():
+        if name == "bandlu_version":
+            continue
+        assert callable(getattr(bandlu, name)), name
