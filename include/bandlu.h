@@ -45,6 +45,8 @@ extern "C" {
 #define BANDLU_ERR_CUDA 1000
 /* a bounded device-side wait gave up; the results of the call are invalid */
 #define BANDLU_ERR_TIMEOUT 1001
+/* dispatch_lu_noalloc: the call would need more scratch than its static array holds */
+#define BANDLU_ERR_SCRATCH 1002
 
 /*
  * detect_bandwidth -- structure identification, step 1 of Sec. II-A; cost
@@ -137,6 +139,33 @@ int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t lda
 int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,
                         int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku,
                         int *d_info, int *d_status, cudaStream_t stream);
+
+/*
+ * dispatch_lu_noalloc -- dispatch_lu for callers that cannot allocate device
+ * memory.  The paper has no counterpart: this is a deployment variant.
+ *
+ * dispatch_lu takes its 8 bytes of scratch (the detected kl, ku) from the
+ * stream-ordered allocator on every call.  Some callers cannot let a library
+ * allocate: a process whose device memory is entirely reserved by its own
+ * caching allocator (an extra allocation can fail or fragment its pool), or a
+ * latency-critical loop whose rules forbid allocation calls, which can take
+ * driver locks or synchronize.  This entry point computes exactly what
+ * dispatch_lu computes, with the same arguments, return codes and outputs, and
+ * calls no cudaMalloc, cudaMallocAsync, cudaFree or other allocating routine.
+ *
+ * Scratch: a file-scope __device__ array of 256 bytes, of which one call uses
+ * 8 (kl, ku), whatever n is; a call needing more returns BANDLU_ERR_SCRATCH.
+ * Every GPU that loads the library holds the array until the process exits.
+ * The first call on each device resolves the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call before
+ * any stream capture.  All calls share the one array and it keeps the last
+ * call's contents (each call clears the pair before detecting), so calls whose
+ * work overlaps on the GPU (different streams or threads, no ordering between
+ * them) race on it: serialise them.
+ * Arguments: as dispatch_lu.
+ */
+int dispatch_lu_noalloc(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *h_kl,
+                        int *h_ku, int *d_info, cudaStream_t stream);
 
 /* Version string of the library build (host, static storage). */
 const char *bandlu_version(void);

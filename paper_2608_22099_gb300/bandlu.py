@@ -18,6 +18,7 @@ BANDLU_OK = 0
 BANDLU_NOT_BANDED = 1
 BANDLU_ERR_CUDA = 1000
 BANDLU_ERR_TIMEOUT = 1001
+BANDLU_ERR_SCRATCH = 1002
 
 _lock = threading.Lock()
 _lib = None
@@ -51,8 +52,10 @@ def load():
         lib.dense_to_band.argtypes = [vp, i64, i64, i32, i32, vp, i64, vp]
         lib.gbtrf.argtypes = [i64, i32, i32, vp, i64, vp, vp, vp]
         lib.dispatch_lu.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
+        lib.dispatch_lu_noalloc.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
         lib.dispatch_lu_batched.argtypes = [vp, i64, i64, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
-        for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "dispatch_lu", "dispatch_lu_batched"):
+        for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "dispatch_lu", "dispatch_lu_batched",
+                  "dispatch_lu_noalloc"):
             getattr(lib, f).restype = ctypes.c_int
         lib.bandlu_version.restype = ctypes.c_char_p
         lib.bandlu_version.argtypes = []
@@ -98,6 +101,15 @@ def dispatch_lu(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -
     kl, ku = ctypes.c_int(-1), ctypes.c_int(-1)
     rc = load().dispatch_lu(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), ctypes.addressof(kl),
                             ctypes.addressof(ku), _ptr(d_info), _stream(stream))
+    return rc, kl.value, ku.value
+
+
+def dispatch_lu_noalloc(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -> tuple[int, int, int]:
+    """dispatch_lu without device allocation (scratch in a static device array).
+    Returns (status, kl, ku)."""
+    kl, ku = ctypes.c_int(-1), ctypes.c_int(-1)
+    rc = load().dispatch_lu_noalloc(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), ctypes.addressof(kl),
+                                    ctypes.addressof(ku), _ptr(d_info), _stream(stream))
     return rc, kl.value, ku.value
 
 

@@ -1,0 +1,77 @@
+// noalloc.cu -- dispatch_lu_noalloc: dispatch_lu without any device allocation.
+//
+// dispatch_lu takes 8 bytes of device scratch per call for the detected (kl, ku)
+// from the stream-ordered allocator.  Some callers cannot allocate device memory
+// from inside a library call: a process whose device memory is entirely reserved
+// by its own caching allocator (an extra cudaMallocAsync can fail or fragment the
+// pool), or a latency-critical loop whose rules forbid allocation calls, which can
+// take driver locks or synchronize.  This entry point keeps that scratch in a
+// file-scope __device__ array instead; every GPU that loads the library holds the
+// array (kNoAllocScratchBytes) until the process exits.
+#include <mutex>
+
+#include "common.cuh"
+
+namespace {
+
+// Scratch of dispatch_lu_noalloc: element 0 = kl, element 1 = ku of the current call.
+// Every call shares it and it keeps the last call's values; the detection launch
+// clears both elements before it folds in the new bandwidths.
+static __device__ __align__(256) int g_noalloc_scratch[64];
+constexpr size_t kNoAllocScratchBytes = sizeof(int) * 64;
+constexpr size_t kNoAllocScratchNeeded = 2 * sizeof(int);  // what one call uses, for every n
+constexpr int kMaxDevices = 64;
+
+std::mutex g_setup_mu;
+int *g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device, resolved once per
+// device with that device current.  Returns nullptr and sets *err on failure.
+int *scratch_for_current_device(int *err) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    *err = BANDLU_ERR_CUDA;
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(g_setup_mu);
+  if (g_scratch_ptr[dev] == nullptr) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
+      *err = BANDLU_ERR_CUDA;
+      return nullptr;
+    }
+    g_scratch_ptr[dev] = static_cast<int *>(p);
+  }
+  return g_scratch_ptr[dev];
+}
+
+}  // namespace
+
+extern "C" int dispatch_lu_noalloc(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv,
+                                   int *h_kl, int *h_ku, int *d_info, cudaStream_t stream) {
+  if (A == nullptr && n > 0) return -1;
+  if (n < 0 || n > (int64_t)INT32_MAX) return -2;
+  if (lda < (n > 1 ? n : 1)) return -3;
+  if (AB == nullptr && n > 0) return -4;
+  if (ldab < 1) return -5;
+  if (ipiv == nullptr && n > 0) return -6;
+  if (h_kl == nullptr) return -7;
+  if (h_ku == nullptr) return -8;
+  if (d_info == nullptr) return -9;
+  if (kNoAllocScratchNeeded > kNoAllocScratchBytes) return BANDLU_ERR_SCRATCH;
+  int err = BANDLU_OK;
+  int *scratch = scratch_for_current_device(&err);
+  if (scratch == nullptr) return err;
+  int rc = bandlu::launch_detect(A, n, lda, scratch, scratch + 1, stream);
+  int h[2] = {0, 0};
+  if (rc == BANDLU_OK && cudaMemcpyAsync(h, scratch, sizeof(h), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    rc = BANDLU_ERR_CUDA;
+  if (cudaStreamSynchronize(stream) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (rc != BANDLU_OK) return rc;
+  *h_kl = h[0];
+  *h_ku = h[1];
+  if (!bandlu::predicate_banded(n, h[0], h[1], ldab)) return BANDLU_NOT_BANDED;
+  rc = bandlu::launch_dense_to_band(A, lda, n, h[0], h[1], AB, ldab, stream);
+  if (rc != BANDLU_OK) return rc;
+  return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream);
+}

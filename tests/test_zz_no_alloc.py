@@ -1,0 +1,46 @@
+"""dispatch_lu_noalloc, the entry point for callers that cannot allocate device
+memory (for example when the process's own caching allocator owns all device
+memory, or a latency-critical loop forbids allocation calls): through the C ABI
+it must give what dispatch_lu gives, on two calls in a row that share its static
+scratch array.  Collected last on purpose."""
+import numpy as np
+import pytest
+import torch
+
+from gpu_helpers import DEV, assert_factor_parity
+from paper_2608_22099_gb300 import bandlu
+from paper_2608_22099_gb300.workloads import make_dense
+
+pytestmark = pytest.mark.gpu
+
+
+def run(fn, A: torch.Tensor, ldab: int):
+    n = A.shape[0]
+    AB = torch.full((n, ldab), -3.0, dtype=torch.float64, device=DEV)
+    ipiv = torch.full((n,), -1, dtype=torch.int32, device=DEV)
+    info = torch.full((1,), -5, dtype=torch.int32, device=DEV)
+    rc, kl, ku = fn(A, n, n, AB, ldab, ipiv, info)
+    torch.cuda.synchronize()
+    return rc, kl, ku, AB.cpu().numpy(), ipiv.cpu().numpy(), int(info.item())
+
+
+def test_noalloc_matches_dispatch_lu_on_two_calls_in_a_row():
+    # the first call leaves a wider band in the shared scratch than the second needs
+    cases = [(make_dense(2048, 20, 9, dist="uniform", seed=71), 2 * 20 + 9 + 1),
+             (make_dense(4096, 16, 16, dist="uniform", seed=1002), 49)]
+    for A, ldab in cases:
+        Ad = A.to(DEV)
+        ref = run(bandlu.dispatch_lu, Ad, ldab)
+        got = run(bandlu.dispatch_lu_noalloc, Ad, ldab)
+        assert got[:3] == ref[:3] and got[0] == 0
+        assert_factor_parity(got[3], got[4], got[5], ref[3], ref[4], ref[5])
+
+
+def test_noalloc_declines_like_dispatch_lu():
+    A = make_dense(1000, 3, 3, dist="uniform", seed=5)
+    A[999, 0] = 1e-3
+    Ad = A.to(DEV)
+    ref = run(bandlu.dispatch_lu, Ad, 10)
+    got = run(bandlu.dispatch_lu_noalloc, Ad, 10)
+    assert got[:3] == ref[:3] == (bandlu.BANDLU_NOT_BANDED, 999, 3)
+    assert np.all(got[3] == -3.0) and np.all(got[4] == -1) and got[5] == -5
