@@ -1,0 +1,34 @@
+/*
+ * bandlu_selftest.h -- self-test hooks of libbandlu.so (not part of the method).
+ *
+ * The pivot chain of gbtrf forms 1/pivot with an integer-pipe reciprocal that
+ * must equal IEEE round-to-nearest division bit for bit (the multipliers are
+ * a * (1/pivot), as DGBTF2 forms them; Sec. III-A names DGBTRF).  These hooks
+ * expose that reciprocal so the test suite can check it against the host's and
+ * the GPU's own division.
+ */
+#ifndef BANDLU_SELFTEST_H
+#define BANDLU_SELFTEST_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* y[i] = reciprocal of x[i] for i < n, computed on the host with the library's
+ * reciprocal.  x and y are HOST arrays of n doubles. */
+void bandlu_selftest_rcp_host(const double *x, double *y, int64_t n);
+
+/* y[i] = 1/x[i] on the device: the library's reciprocal (use_division == 0) or
+ * the compiler's double division (use_division != 0), for comparison.  x and y
+ * are DEVICE arrays of n doubles; asynchronous on `stream`.
+ * Returns 0, -1 (x null), -2 (y null), -3 (n < 0) or BANDLU_ERR_CUDA. */
+int bandlu_selftest_rcp_device(const double *x, double *y, int64_t n, int use_division, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BANDLU_SELFTEST_H */

@@ -57,6 +57,10 @@ def load():
         for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "dispatch_lu", "dispatch_lu_batched",
                   "dispatch_lu_noalloc"):
             getattr(lib, f).restype = ctypes.c_int
+        lib.bandlu_selftest_rcp_host.argtypes = [vp, vp, i64]
+        lib.bandlu_selftest_rcp_host.restype = None
+        lib.bandlu_selftest_rcp_device.argtypes = [vp, vp, i64, i32, vp]
+        lib.bandlu_selftest_rcp_device.restype = ctypes.c_int
         lib.bandlu_version.restype = ctypes.c_char_p
         lib.bandlu_version.argtypes = []
         _lib = lib
@@ -118,6 +122,24 @@ def dispatch_lu_batched(A, n: int, lda: int, strideA: int, batch: int, AB, ldab:
     return load().dispatch_lu_batched(_ptr(A), n, lda, strideA, batch, _ptr(AB), ldab, strideAB, _ptr(ipiv),
                                       strideP, _ptr(d_kl), _ptr(d_ku), _ptr(d_info), _ptr(d_status),
                                       _stream(stream))
+
+
+def bandlu_selftest_rcp_host(x, y, n: int) -> None:
+    """Self-test hook: the library's reciprocal on the host (x, y: host buffers of n doubles)."""
+    load().bandlu_selftest_rcp_host(_ptr_host(x), _ptr_host(y), n)
+
+
+def bandlu_selftest_rcp_device(x, y, n: int, use_division: int, stream=None) -> int:
+    """Self-test hook: the library's reciprocal (or plain division) on the device."""
+    return load().bandlu_selftest_rcp_device(_ptr(x), _ptr(y), n, use_division, _stream(stream))
+
+
+def _ptr_host(x) -> int:
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "ctypes"):
+        return int(x.ctypes.data)
+    return int(x.data_ptr())
 
 
 def check(rc: int, what: str = "call") -> int:

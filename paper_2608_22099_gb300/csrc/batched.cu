@@ -14,6 +14,7 @@
 #include <climits>
 
 #include "common.cuh"
+#include "rcp.cuh"
 
 namespace bandlu {
 namespace {
@@ -144,7 +145,7 @@ __device__ int warp_gbtrf(double *ab, long long ldab, long long n, int kl, int k
         __syncwarp();
       }
       if (km > 0) {
-        const double r = 1.0 / pv;
+        const double r = rcp_rn(pv);  // IEEE 1/pv on the integer pipes
         for (long long t = 1 + lane; t <= km; t += 32) col[kv + t] *= r;
         __syncwarp();
         const long long tot = (ju - j) * km;

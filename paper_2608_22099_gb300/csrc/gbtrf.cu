@@ -15,10 +15,7 @@
 //    can start at once.  Warps 1..3 (updaters) apply step j to columns
 //    j+2..j+kv (column j+2 first, which the panel needs next), stream the
 //    finished U row to global memory and prefetch the rows that enter the
-//    window.  Hand-offs use mbarriers with bounded waits:
-//      full[b]   panel -> updaters: step j's multipliers, row slots, zero-pivot flag
-//      empty[b]  updaters -> panel and updaters: all updater warps finished step j
-//      colready  warp 1 -> panel: column j+2 holds step j (and column j+1+kv is cleared)
+//    window.  Hand-offs are two named barriers per step (see kBarPub/kBarCol).
 //
 //  * k_gbtrf_generic (any kl, ku).  One CTA works directly on AB in global
 //    memory (the active window stays L2-resident), one column at a time.
@@ -32,30 +29,54 @@
 #include <climits>
 
 #include "common.cuh"
-#include "sync.cuh"
+#include "rcp.cuh"
 
 namespace bandlu {
 namespace {
 
 constexpr int kDelta = 4;          // rows prefetched ahead of the active window
 constexpr int kWinMaxKl = 31 - kDelta;
-constexpr int kNU = 3;             // updater warps
+constexpr int kWarps = 16;         // warp 0 panel, warp 4 row prefetch, 12 updaters
+constexpr int kNU = 12;            // updater warps: every warp w with w % 4 != 0
 constexpr int kNUT = 32 * kNU;     // updater threads
+constexpr int kPrefetchWarp = 4;
 
-struct WinShared {
-  unsigned long long full[2];   // panel -> updaters: step buffer b is published
-  unsigned long long empty[2];  // updaters -> panel: step buffer b is consumed
-  unsigned long long colready;  // warp 1 -> panel: column j+2 holds step j
-  int abort_flag;
-  int zp[2];
-  int slot[2][32];
-  double l[2][32];
+// One published row of step j: its multiplier and the offset of its slot in W.
+struct __align__(16) RowPk {
+  double l;
+  int rb;   // slot * CS
+  int pad;
 };
 
-template <int PF>
-__global__ void __launch_bounds__(128, 1) k_gbtrf_window(long long n, int kl, int ku, double *__restrict__ AB,
-                                                          long long ldab, int *__restrict__ ipiv,
-                                                          int *__restrict__ d_info) {
+struct WinShared {
+  int zp[2];
+  RowPk pk[2][32];
+};
+
+// Named barriers of the window kernel (0 is __syncthreads):
+//   kBarPub: the panel arrives once step j's multipliers, row slots and zero-pivot
+//            flag are published; the 12 updater warps and the prefetch warp sync
+//            on it, so it also orders all their step j-1 work before any step j.
+//   kBarCol: warp 1 arrives once column j+2 holds step j (and column j+1+kv is
+//            cleared); the panel syncs on it before it reads column j+2.
+// Every participating warp runs exactly n steps and executes its barrier
+// operations unconditionally, once per step.  The panel arrives at kBarPub(j)
+// only after kBarCol(j-1), which warp 1 reaches only after kBarPub(j-1)
+// completed, and warp 1 arrives at kBarCol(j) only after kBarPub(j) completed,
+// which needs the panel's arrival after kBarCol(j-1): the phases alternate.
+constexpr int kBarPub = 1, kBarCol = 2;
+constexpr int kPubCount = 32 * (1 + kNU + 1);
+__device__ __forceinline__ void bar_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+__device__ __forceinline__ void bar_arrive(int id, int count) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+template <int K, int PF>
+__global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, int ku, double *__restrict__ AB,
+                                                                  long long ldab, int *__restrict__ ipiv,
+                                                                  int *__restrict__ d_info) {
   extern __shared__ double W[];  // R * CS
   __shared__ WinShared sh;
   const int kv = kl + ku;
@@ -63,14 +84,6 @@ __global__ void __launch_bounds__(128, 1) k_gbtrf_window(long long n, int kl, in
   const int CS = kl + kv + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  if (threadIdx.x == 0) {
-    mbar_init(&sh.full[0], 1);
-    mbar_init(&sh.full[1], 1);
-    mbar_init(&sh.empty[0], kNU);
-    mbar_init(&sh.empty[1], kNU);
-    mbar_init(&sh.colready, 1);
-    sh.abort_flag = 0;
-  }
   // Fill-row entries of the top-left corner (element row < 0) are cleared, as
   // the elimination clears every fill row before it starts.
   for (int e = threadIdx.x; e < kl * kv; e += blockDim.x) {
@@ -78,13 +91,13 @@ __global__ void __launch_bounds__(128, 1) k_gbtrf_window(long long n, int kl, in
     if (c < kv - r && c < n) AB[r + (long long)c * ldab] = 0.0;
   }
   // Rows 0..R-1 go to slots 0..R-1; row i covers columns i-kl .. i+kv.
-  const int R0 = (int)min((long long)R, n);
+  const int R0 = min(R, n);
   for (int e = threadIdx.x; e < R0 * CS; e += blockDim.x) {
     const int i = e / CS, k = e - i * CS;
-    const long long c = (long long)i - kl + k;
+    const int c = i - kl + k;
     double v = 0.0;
-    if (c >= 0 && c < n && c <= i + ku) v = AB[(kv + i - c) + c * ldab];
-    const int q = (int)(((c % CS) + CS) % CS);
+    if (c >= 0 && c < n && c <= i + ku) v = AB[(kv + i - c) + (long long)c * ldab];
+    const int q = ((c % CS) + CS) % CS;
     W[i * CS + q] = v;
   }
   __syncthreads();
@@ -95,12 +108,12 @@ __global__ void __launch_bounds__(128, 1) k_gbtrf_window(long long n, int kl, in
     int slot_reg = lane;  // slot of logical row j+lane (lanes < R)
     double cur = (lane <= kl && lane < n) ? W[lane * CS] : 0.0;
     int qn = 1 % CS;  // column slot of column j+1
-    for (long long j = 0; j < n; ++j) {
-      const int km = (int)min((long long)kl, n - 1 - j);
+    for (int j = 0; j < n; ++j) {
+      const int km = min(kl, n - 1 - j);
       const bool valid = lane <= km;
       const unsigned long long key = valid ? abs_key(cur) : 0ull;
-      // Every candidate's reciprocal is formed while the argmax runs.
-      const double rl = 1.0 / ((valid && nz(cur)) ? cur : 1.0);
+      // Every candidate's reciprocal is formed (integer pipes) while the argmax runs.
+      const double rl = rcp_rn((valid && nz(cur)) ? cur : 1.5);
       const int p = warp_argmax_first(key);
       const double pv = __shfl_sync(FULL, cur, p);
       const double r = __shfl_sync(FULL, rl, p);
@@ -112,64 +125,112 @@ __global__ void __launch_bounds__(128, 1) k_gbtrf_window(long long n, int kl, in
       const int sp = __shfl_sync(FULL, slot_reg, p);
       if (lane == p) slot_reg = s0;
       if (lane == 0) slot_reg = sp;
+      // column j+1, logical rows j .. j+kl+1 (holds steps <= j-1)
+      if (j >= 1) bar_sync(kBarCol, 64);
+      double v = 0.0;
+      if (j + 1 < n && lane <= kl + 1 && j + lane < n) v = W[slot_reg * CS + qn];
+      // U(j, j+1); when kv == 0 (diagonal matrix) column j+1 lies outside row j's band
+      const double u = kv >= 1 ? __shfl_sync(FULL, v, 0) : 0.0;
       const double l = (!zp && lane >= 1 && valid) ? cur * r : cur;
-      if (lane == 0) {
-        ipiv[j] = (int)(j + p + 1);
-        AB[kv + j * ldab] = pv;
-      }
-      if (lane >= 1 && valid) AB[(kv + lane) + j * ldab] = l;
-      if (zp && info == 0) info = (int)(j + 1);
-      const int b = (int)(j & 1);
-      if (j >= 1 && !mbar_wait_warp(&sh.colready, (unsigned)((j - 1) & 1), &sh.abort_flag)) break;
-      if (j >= 2 && !mbar_wait_warp(&sh.empty[b], (unsigned)(((j - 2) >> 1) & 1), &sh.abort_flag)) break;
-      sh.l[b][lane] = l;
-      sh.slot[b][lane] = slot_reg;
+      // buffer b was last read in step j-2, which every updater finished before
+      // warp 1 reached kBarCol(j-1)
+      const int b = j & 1;
+      sh.pk[b][lane].l = l;
+      sh.pk[b][lane].rb = slot_reg * CS;
       if (lane == 0) sh.zp[b] = zp ? 1 : 0;
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sh.full[b]);
+      bar_arrive(kBarPub, kPubCount);
       if (j + 1 < n) {
-        // column j+1, logical rows j .. j+kl+1 (holds steps <= j-1)
-        double v = 0.0;
-        if (lane <= kl + 1 && j + lane < n) v = W[slot_reg * CS + qn];
-        // U(j, j+1); when kv == 0 (diagonal matrix) column j+1 lies outside row j's band
-        const double u = kv >= 1 ? __shfl_sync(FULL, v, 0) : 0.0;
-        if (lane == 0 && kv >= 1) AB[(kv - 1) + (j + 1) * ldab] = u;
         if (!zp && nz(u) && lane >= 1 && valid) v = fma(-l, u, v);
         cur = __shfl_down_sync(FULL, v, 1);  // logical rows j+1 .. j+1+kl
       }
+      if (lane == 0) {
+        ipiv[j] = j + p + 1;
+        AB[kv + j * ldab] = pv;
+        if (kv >= 1 && j + 1 < n) AB[(kv - 1) + (j + 1) * ldab] = u;
+      }
+      if (lane >= 1 && valid) AB[(kv + lane) + j * ldab] = l;
+      if (zp && info == 0) info = j + 1;
       const int sfirst = __shfl_sync(FULL, slot_reg, 0);
       const int sn = __shfl_down_sync(FULL, slot_reg, 1);
       slot_reg = (lane == R - 1) ? sfirst : sn;  // retired row's slot takes row j+R
       qn = (qn + 1 == CS) ? 0 : qn + 1;
     }
-  } else if (warp <= kNU) {
-    // ---------------- updater warps ----------------
-    const int tid_u = threadIdx.x - 32;
+    bar_sync(kBarCol, 64);  // warp 1's arrival of the last step
+  } else if (warp == kPrefetchWarp) {
+    // ---------------- row prefetch warp ----------------
+    // Row j-1+R enters the slot that row j-1 left; it is fetched in step j and
+    // stored in step j+1 (a whole step for the global loads to land).
+    int pfo[PF];
+#pragma unroll
+    for (int k = 0; k < PF; ++k) pfo[k] = (kDelta + lane + 32 * k) % CS;
     double pf[PF];
     bool have_pf = false;
-    long long pf_row = 0;
-    int pf_slot = 0;
+    int pf_rb = 0, pf_q = 0;
+    int qj = 0;
+    for (int j = 0; j < n; ++j) {
+      const int b = j & 1;
+      bar_sync(kBarPub, kPubCount);
+      if (have_pf) {
+#pragma unroll
+        for (int k = 0; k < PF; ++k) {
+          if (lane + 32 * k < CS) {
+            int q = pf_q + pfo[k];
+            if (q >= CS) q -= CS;
+            W[pf_rb + q] = pf[k];
+          }
+        }
+        have_pf = false;
+      }
+      if (j >= 1 && j - 1 + R < n) {
+        const int i = j - 1 + R;
+        pf_rb = sh.pk[b][R - 1].rb;
+        pf_q = qj;
+        have_pf = true;
+#pragma unroll
+        for (int k = 0; k < PF; ++k) {
+          const int kk = lane + 32 * k;
+          const int c = i - kl + kk;
+          pf[k] = (kk < CS && c <= i + ku && c < n) ? AB[(kv + i - c) + (long long)c * ldab] : 0.0;
+        }
+      }
+      qj = (qj + 1 == CS) ? 0 : qj + 1;
+    }
+  } else if ((warp & 3) != 0) {
+    // ---------------- updater warps ----------------
+    const int uw = warp - 1 - (warp >> 2);  // 0..kNU-1
+    const int tid_u = uw * 32 + lane;
+    const int rows = kl + 1;
+    const int E = kv > 2 ? (kv - 2) * rows : 0;
+    // Static element map of columns j+3..j+kv: element e -> column offset
+    // d = 3 + e / rows, row offset t = e % rows (t = 0: the U row is written out).
+    int ed[K], et[K];
+    long long uoff[K];  // offset of U(j, j+d) in AB relative to column j
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+      const int e = tid_u + kNUT * k;
+      ed[k] = e < E ? 3 + e / rows : 0;
+      et[k] = e < E ? e - (ed[k] - 3) * rows : 0;
+      uoff[k] = (kv - ed[k]) + (long long)ed[k] * ldab;
+    }
     int qj = 0;  // column slot of column j
-    for (long long j = 0; j < n; ++j) {
-      const int b = (int)(j & 1);
-      if (!mbar_wait_warp(&sh.full[b], (unsigned)((j >> 1) & 1), &sh.abort_flag)) break;
-      // Consecutive steps update the same entries through different threads: every
-      // updater warp must have finished step j-1 before any starts step j.
-      if (j >= 1 && !mbar_wait_warp(&sh.empty[b ^ 1], (unsigned)(((j - 1) >> 1) & 1), &sh.abort_flag)) break;
-      const int km = (int)min((long long)kl, n - 1 - j);
+    for (int j = 0; j < n; ++j) {
+      const int b = j & 1;
+      bar_sync(kBarPub, kPubCount);
+      const int km = min(kl, n - 1 - j);
       const bool zp = sh.zp[b] != 0;
-      const long long cmax = min(j + kv, n - 1);
-      const int s0 = sh.slot[b][0];
+      const int cmax = min(j + kv, n - 1);
+      const int rb0 = sh.pk[b][0].rb;
       if (warp == 1) {
-        const long long c = j + 2;
+        const int c = j + 2;
         if (c <= cmax) {
           int q = qj + 2;
           if (q >= CS) q -= CS;
-          const double u = W[s0 * CS + q];
-          if (lane == 0) AB[(kv - 2) + c * ldab] = u;
+          const double u = W[rb0 + q];
+          if (lane == 0) AB[(kv - 2) + (long long)c * ldab] = u;
           if (!zp && nz(u) && lane >= 1 && lane <= km) {
-            const int st = sh.slot[b][lane];
-            W[st * CS + q] = fma(-sh.l[b][lane], u, W[st * CS + q]);
+            const RowPk pk = sh.pk[b][lane];
+            W[pk.rb + q] = fma(-pk.l, u, W[pk.rb + q]);
           }
         }
         // Column j+1+kv enters the window at step j+1.  Rows j+1..j+kl (any
@@ -178,59 +239,44 @@ __global__ void __launch_bounds__(128, 1) k_gbtrf_window(long long n, int kl, in
         if (lane >= 1 && lane <= kl && j + 1 + kv < n) {
           int qe = qj + 1 + kv;
           if (qe >= CS) qe -= CS;
-          W[sh.slot[b][lane] * CS + qe] = 0.0;
+          W[sh.pk[b][lane].rb + qe] = 0.0;
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sh.colready);
+        bar_arrive(kBarCol, 64);
       }
-      const long long ncols = cmax - (j + 2);
-      if (ncols > 0) {
-        const int rows = km + 1;
-        const int tot = (int)ncols * rows;
-        for (int e = tid_u; e < tot; e += kNUT) {
-          const int cc = e / rows, t = e - cc * rows;
-          const long long c = j + 3 + cc;
-          int q = qj + 3 + cc;
-          if (q >= CS) q -= CS;
-          const double u = W[s0 * CS + q];
-          if (t == 0) {
-            AB[(kv + j - c) + c * ldab] = u;  // U(j, c)
-          } else if (!zp && nz(u)) {
-            const int st = sh.slot[b][t];
-            W[st * CS + q] = fma(-sh.l[b][t], u, W[st * CS + q]);
-          }
-        }
-      }
-      // The row fetched one step ago goes into its slot (the slot's previous
-      // row retired two steps ago).
-      if (have_pf) {
+      // columns j+3..j+kv: all loads first, then the fused multiply-adds, then the stores
+      const bool full = j + kv <= n - 1;  // every mapped element is inside the matrix
+      double *ABj = AB + (long long)j * ldab;
+      double uu[K], xx[K], ll[K];
+      int rr[K], qq[K];
+      bool act[K];
 #pragma unroll
-        for (int k = 0; k < PF; ++k) {
-          const int kk = tid_u + k * kNUT;
-          if (kk < CS) W[pf_slot * CS + (int)((pf_row - kl + kk) % CS)] = pf[k];
-        }
-        have_pf = false;
+      for (int k = 0; k < K; ++k) {
+        act[k] = ed[k] != 0 && (full || (j + ed[k] <= cmax && et[k] <= km));
+        int q = qj + ed[k];
+        if (q >= CS) q -= CS;
+        qq[k] = q;
+        uu[k] = act[k] ? W[rb0 + q] : 0.0;
+        const RowPk pk = sh.pk[b][et[k]];
+        ll[k] = pk.l;
+        rr[k] = pk.rb;
       }
-      // Fetch row j-1+R: its band entries, zeros for the rest of its columns.
-      if (j >= 1 && j - 1 + R < n) {
-        const long long i = j - 1 + R;
-        pf_row = i;
-        pf_slot = sh.slot[b][R - 1];
-        have_pf = true;
 #pragma unroll
-        for (int k = 0; k < PF; ++k) {
-          const int kk = tid_u + k * kNUT;
-          const long long c = i - kl + kk;
-          pf[k] = (kk < CS && c <= i + ku && c < n) ? AB[(kv + i - c) + c * ldab] : 0.0;
+      for (int k = 0; k < K; ++k) xx[k] = (act[k] && et[k] > 0) ? W[rr[k] + qq[k]] : 0.0;
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        if (!act[k]) continue;
+        if (et[k] == 0) {
+          ABj[uoff[k]] = uu[k];  // U(j, j+d)
+        } else if (!zp && nz(uu[k])) {
+          W[rr[k] + qq[k]] = fma(-ll[k], uu[k], xx[k]);
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sh.empty[b]);
       qj = (qj + 1 == CS) ? 0 : qj + 1;
     }
   }
   __syncthreads();
-  if (threadIdx.x == 0) *d_info = sh.abort_flag ? -BANDLU_ERR_TIMEOUT : info;
+  if (threadIdx.x == 0) *d_info = info;
 }
 
 __global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int ku, double *__restrict__ AB,
@@ -302,19 +348,28 @@ __global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int
   if (tid == 0) *d_info = info;
 }
 
-template <int PF>
+template <int K, int PF>
 int launch_window(long long n, int kl, int ku, double *AB, long long ldab, int *ipiv, int *d_info, size_t smem,
                   cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    if (cudaFuncSetAttribute(k_gbtrf_window<PF>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
+    if (cudaFuncSetAttribute(k_gbtrf_window<K, PF>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
         cudaSuccess)
       return BANDLU_ERR_CUDA;
     attr = true;
   }
-  k_gbtrf_window<PF><<<1, 128, smem, s>>>(n, kl, ku, AB, ldab, ipiv, d_info);
+  k_gbtrf_window<K, PF><<<1, kWarps * 32, smem, s>>>((int)n, kl, ku, AB, ldab, ipiv, d_info);
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;
+}
+
+template <int K>
+int launch_window_pf(int pf, long long n, int kl, int ku, double *AB, long long ldab, int *ipiv, int *d_info,
+                     size_t smem, cudaStream_t s) {
+  if (pf <= 1) return launch_window<K, 1>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+  if (pf <= 2) return launch_window<K, 2>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+  if (pf <= 4) return launch_window<K, 4>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+  return launch_window<K, 8>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
 }
 
 }  // namespace
@@ -328,12 +383,14 @@ int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv,
   const long long CS = kl + kv + 1;
   const long long R = kl + 1 + kDelta;
   const size_t smem = (size_t)(R * CS) * sizeof(double);
-  if (kl <= kWinMaxKl && CS <= 8 * kNUT && smem <= 200 * 1024) {
-    const int pf = (int)((CS + kNUT - 1) / kNUT);
-    if (pf <= 1) return launch_window<1>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
-    if (pf <= 2) return launch_window<2>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
-    if (pf <= 4) return launch_window<4>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
-    return launch_window<8>(n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+  const long long E = kv > 2 ? (kv - 2) * (kl + 1) : 0;  // trailing elements per step
+  if (kl <= kWinMaxKl && CS <= 8 * 32 && E <= 8 * kNUT && smem <= 200 * 1024) {
+    const int pf = (int)((CS + 31) / 32);
+    const int k = (int)((E + kNUT - 1) / kNUT);
+    if (k <= 1) return launch_window_pf<1>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+    if (k <= 2) return launch_window_pf<2>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+    if (k <= 4) return launch_window_pf<4>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+    return launch_window_pf<8>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
   }
   k_gbtrf_generic<<<1, 1024, 0, s>>>(n, kl, ku, AB, ldab, ipiv, d_info);
   BANDLU_CHECK_LAUNCH();

@@ -1,0 +1,105 @@
+// rcp.cuh -- correctly rounded double reciprocal on the integer and FP32 pipes.
+//
+// GB300's FP64 pipe issues one warp instruction per 64 clocks per SMSP, so the
+// ~7 dependent FP64 operations of a double division sit squarely on the pivot
+// chain of the band LU.  This reciprocal uses integer arithmetic instead.  For a
+// normal b = +-m * 2^(E-1075) with 2^52 <= m < 2^53 (E the biased exponent),
+//   1/b = (2^105 / m) * 2^(970-E),
+// so the rounded significand is q = Q + [2R > m] where Q = floor(2^105/m) and
+// R = 2^105 - Q*m (no ties are possible: 2^106/m is not an integer for m > 2^52).
+// Q is found as a quotient by approximate reciprocal with remainder correction
+// (Knuth, TAOCP Vol. 2, Sec. 4.3.1): a Newton step on a two-float (double-float)
+// representation of m gives Q within 2^8; one correction Q += (2^105 - Q*m)/m,
+// estimated in single precision from the exact 64-bit remainder, brings Q within
+// one unit; the exact remainder then fixes Q and decides the rounding.
+// The result is the IEEE round-to-nearest 1/b, bit for bit.  Zeros, subnormals,
+// infinities, NaN and |b| >= 2^1021 (whose reciprocal is subnormal) go to the
+// ordinary division.
+#pragma once
+
+#include <cstdint>
+#include <cstring>
+
+namespace bandlu {
+
+__host__ __device__ __forceinline__ float rcp_approx_f32(float x) {
+#ifdef __CUDA_ARCH__
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+#else
+  return 1.0f / x;
+#endif
+}
+
+__host__ __device__ __forceinline__ uint64_t dbits(double x) {
+#ifdef __CUDA_ARCH__
+  return (uint64_t)__double_as_longlong(x);
+#else
+  uint64_t u;
+  std::memcpy(&u, &x, 8);
+  return u;
+#endif
+}
+
+__host__ __device__ __forceinline__ double bitsd(uint64_t u) {
+#ifdef __CUDA_ARCH__
+  return __longlong_as_double((long long)u);
+#else
+  double x;
+  std::memcpy(&x, &u, 8);
+  return x;
+#endif
+}
+
+__host__ __device__ __forceinline__ uint32_t fbits(float x) {
+#ifdef __CUDA_ARCH__
+  return (uint32_t)__float_as_uint(x);
+#else
+  uint32_t u;
+  std::memcpy(&u, &x, 4);
+  return u;
+#endif
+}
+
+// Correctly rounded 1/b (IEEE binary64, round to nearest even).
+__host__ __device__ __forceinline__ double rcp_rn(double b) {
+  const uint64_t bits = dbits(b);
+  const uint64_t E = (bits >> 52) & 0x7ffull;
+  const uint64_t frac = bits & ((1ull << 52) - 1);
+  const uint64_t sign = bits & (1ull << 63);
+  if (E == 0 || E >= 2045) return 1.0 / b;
+  if (frac == 0) return bitsd(sign | ((2046 - E) << 52));  // power of two: exact
+  const uint64_t m = frac | (1ull << 52);
+  // M = m / 2^29 = xh + xl/2^29 with xh the 24-bit rounding (exact in single
+  // precision) and |xl| <= 2^28.
+  const uint32_t xh = (uint32_t)(((m >> 28) + 1) >> 1);
+  const int32_t xl = (int32_t)((int64_t)m - ((int64_t)xh << 29));
+  const float xhf = (float)xh, xlf = (float)xl * 0x1p-29f;
+  // y ~ 1/xh: hardware seed plus one Newton step; then one Newton step for 1/M
+  // carried as the unevaluated pair y + t (relative error below 2^-45).
+  const float y0 = rcp_approx_f32(xhf);
+  const float y = fmaf(y0, fmaf(-xhf, y0, 1.0f), y0);
+  const float e = fmaf(-xlf, y, fmaf(-xhf, y, 1.0f));  // 1 - M*y
+  const float t = y * e;
+  // Q = (y + t) * 2^76 ~ 2^105/m within 2^8; y*2^76 is an exact integer (y in [2^-24, 2^-23]).
+  const uint32_t yb = fbits(y);
+  uint64_t Q = (uint64_t)((yb & 0x7fffffu) | 0x800000u) << (int)((yb >> 23) - 74u);
+  Q = (uint64_t)((int64_t)Q + (int64_t)(int32_t)(t * 0x1p76f));
+  // one correction from the exact remainder: 2^105 = 0 mod 2^64 and |R| < 2^62
+  int64_t R = (int64_t)(0ull - Q * m);
+  Q = (uint64_t)((int64_t)Q + (int64_t)(int32_t)((float)(int32_t)(R >> 31) * y * 4.0f));
+  // now |Q - 2^105/m| < 1.01: the exact remainder fixes Q and decides the rounding
+  R = (int64_t)(0ull - Q * m);
+  if (R < 0) {
+    Q -= 1;
+    R += (int64_t)m;
+  } else if (R >= (int64_t)m) {
+    Q += 1;
+    R -= (int64_t)m;
+  }
+  if ((uint64_t)R > m - (uint64_t)R) Q += 1;  // 2R > m: round up
+  return bitsd(sign | ((2045 - E) << 52) | (Q - (1ull << 52)));
+}
+
+}  // namespace bandlu

@@ -1,0 +1,40 @@
+// selftest.cu -- self-test hooks (declared in include/bandlu_selftest.h): the
+// integer-pipe reciprocal used on the pivot chain, callable on the host and on
+// the device so tests can compare it bit for bit with IEEE division.
+#include "bandlu_selftest.h"
+#include "common.cuh"
+#include "rcp.cuh"
+
+namespace {
+__global__ void k_rcp(const double *__restrict__ x, double *__restrict__ y, long long n) {
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
+    y[i] = bandlu::rcp_rn(x[i]);
+}
+__global__ void k_div(const double *__restrict__ x, double *__restrict__ y, long long n) {
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
+    y[i] = 1.0 / x[i];
+}
+}  // namespace
+
+extern "C" {
+
+void bandlu_selftest_rcp_host(const double *x, double *y, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) y[i] = bandlu::rcp_rn(x[i]);
+}
+
+int bandlu_selftest_rcp_device(const double *x, double *y, int64_t n, int use_division, cudaStream_t stream) {
+  if (n < 0) return -3;
+  if (n == 0) return BANDLU_OK;
+  if (x == nullptr) return -1;
+  if (y == nullptr) return -2;
+  long long blocks = (n + 255) / 256;
+  if (blocks > 152ll * 64) blocks = 152ll * 64;
+  if (use_division)
+    k_div<<<(unsigned)blocks, 256, 0, stream>>>(x, y, n);
+  else
+    k_rcp<<<(unsigned)blocks, 256, 0, stream>>>(x, y, n);
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+}  // extern "C"

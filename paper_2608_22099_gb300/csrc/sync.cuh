@@ -45,16 +45,24 @@ __device__ __forceinline__ bool mbar_try_wait(unsigned long long *bar, unsigned 
 // 32 lanes of a warp; the result is warp-uniform.
 __device__ __forceinline__ bool mbar_wait_warp(unsigned long long *bar, unsigned parity, volatile int *abort_flag) {
   bool ok = true;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (*abort_flag) { ok = false; break; }
-    if (clock64() - t0 > kWaitLimitCycles) {
-      *abort_flag = 1;
-      ok = false;
-      break;
+  if (!mbar_try_wait(bar, parity)) {
+    const long long t0 = clock64();
+    for (unsigned it = 1;; ++it) {
+      if (mbar_try_wait(bar, parity)) break;
+      if ((it & 31u) == 0) {
+        if (*abort_flag) {
+          ok = false;
+          break;
+        }
+        if (clock64() - t0 > kWaitLimitCycles) {
+          *abort_flag = 1;
+          ok = false;
+          break;
+        }
+      }
     }
   }
-  return __all_sync(0xffffffffu, ok);
+  return __all_sync(0xffffffffu, ok);  // one call site: lanes reconverge here
 }
 
 }  // namespace bandlu
