@@ -38,10 +38,13 @@ def load():
     with _lock:
         if _lib is not None:
             return _lib
-        path = _build.LIB
-        if not _build.up_to_date():
+        # BANDLU_CHECKED=1 selects the checked build (bounded inter-warp waits) for
+        # development runs; the default is the production library.
+        checked = os.environ.get("BANDLU_CHECKED", "") == "1"
+        path = _build.CHECKED_LIB if checked else _build.LIB
+        if not _build.up_to_date(path):
             try:
-                path = _build.build()
+                path = _build.build(checked=checked)
             except Exception as e:  # noqa: BLE001 - re-raised with context
                 raise BandLUError(f"the CUDA library could not be built: {e}") from e
         if not os.path.exists(path):

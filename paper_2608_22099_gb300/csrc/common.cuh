@@ -32,6 +32,17 @@ __device__ __forceinline__ int warp_argmax_first(unsigned long long key) {
   return __ffs(win) - 1;
 }
 
+// As warp_argmax_first, and *all_zero tells whether every key is zero.
+__device__ __forceinline__ int warp_argmax_first_z(unsigned long long key, bool *all_zero) {
+  const unsigned hi = (unsigned)(key >> 32), lo = (unsigned)key;
+  const unsigned mhi = __reduce_max_sync(FULL, hi);
+  const unsigned lo2 = (hi == mhi) ? lo : 0u;
+  const unsigned mlo = __reduce_max_sync(FULL, lo2);
+  const unsigned win = __ballot_sync(FULL, hi == mhi && lo == mlo);
+  *all_zero = (mhi | mlo) == 0u;
+  return __ffs(win) - 1;
+}
+
 // (key, index) pair that prefers the larger key and, on a tie, the smaller index.
 struct KeyIdx {
   unsigned long long key;

@@ -30,48 +30,102 @@
 
 #include "common.cuh"
 #include "rcp.cuh"
+#include "sync.cuh"
 
 namespace bandlu {
 namespace {
 
 constexpr int kDelta = 4;          // rows prefetched ahead of the active window
 constexpr int kWinMaxKl = 31 - kDelta;
-constexpr int kWarps = 16;         // warp 0 panel, warp 4 row prefetch, 12 updaters
-constexpr int kNU = 12;            // updater warps: every warp w with w % 4 != 0
+constexpr int kWarps = 16;         // warp 0 panel, 4 helper, 13 I/O, 11 updaters, 8 and 12 idle
+constexpr int kNU = 11;            // updater warps: every warp w with w % 4 != 0 except kIoWarp
 constexpr int kNUT = 32 * kNU;     // updater threads
-constexpr int kPrefetchWarp = 4;
+constexpr int kHelperWarp = 4;     // shares the panel's SMSP (shared-memory work only)
+constexpr int kIoWarp = 13;        // global stores and row prefetch, away from the panel's SMSP
 
-// One published row of step j: its multiplier and the offset of its slot in W.
+// One published row of step j: its multiplier (the pivot itself for row 0) and
+// the offset of its slot in W.
 struct __align__(16) RowPk {
   double l;
   int rb;   // slot * CS
   int pad;
 };
 
-struct WinShared {
-  int zp[2];
-  RowPk pk[2][32];
+struct __align__(16) StepMeta {
+  double u1;  // U(j, j+1)
+  int zp;     // exact zero pivot
+  int p;      // pivot offset
 };
 
+
 // Named barriers of the window kernel (0 is __syncthreads):
-//   kBarPub: the panel arrives once step j's multipliers, row slots and zero-pivot
-//            flag are published; the 12 updater warps and the prefetch warp sync
-//            on it, so it also orders all their step j-1 work before any step j.
-//   kBarCol: warp 1 arrives once column j+2 holds step j (and column j+1+kv is
-//            cleared); the panel syncs on it before it reads column j+2.
+//   kBarPub: the panel arrives once step j (multipliers, row slots, pivot) is
+//            published; the 12 updater warps and the helper warp sync on it, so
+//            it also orders all their step j-1 work before any step j.
+//   kBarCol: the helper warp arrives once column j+2 holds step j (and column
+//            j+1+kv is cleared); the panel syncs on it before it reads column j+2.
 // Every participating warp runs exactly n steps and executes its barrier
 // operations unconditionally, once per step.  The panel arrives at kBarPub(j)
-// only after kBarCol(j-1), which warp 1 reaches only after kBarPub(j-1)
-// completed, and warp 1 arrives at kBarCol(j) only after kBarPub(j) completed,
-// which needs the panel's arrival after kBarCol(j-1): the phases alternate.
+// only after kBarCol(j-1), which the helper reaches only after kBarPub(j-1)
+// completed, and the helper arrives at kBarCol(j) only after kBarPub(j)
+// completed, which needs the panel's arrival after kBarCol(j-1): the phases of
+// both barriers alternate.
 constexpr int kBarPub = 1, kBarCol = 2;
-constexpr int kPubCount = 32 * (1 + kNU + 1);
-__device__ __forceinline__ void bar_sync(int id, int count) {
+constexpr int kPubCount = 32 * (1 + kNU + 2);
+
+#ifdef BANDLU_BOUNDED_SYNC
+// Checked build (development and tests only): the same protocol on mbarriers
+// with bounded waits.  A protocol slip (a missing participant, a miscounted
+// barrier) ends the kernel with info = -BANDLU_ERR_TIMEOUT instead of a hang.
+struct BarState {
+  unsigned long long mb[3];
+  int abort_flag;
+};
+__device__ __forceinline__ void bar_init(BarState &st) {
+  mbar_init(&st.mb[kBarPub], kPubCount / 32);
+  mbar_init(&st.mb[kBarCol], 2);
+  st.abort_flag = 0;
+}
+__device__ __forceinline__ void bar_arrive_x(BarState &st, int id) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(&st.mb[id]);
+}
+// phase: how many times this warp has synced on barrier `id` so far
+__device__ __forceinline__ bool bar_sync_x(BarState &st, int id, unsigned &phase) {
+  bar_arrive_x(st, id);
+  const bool ok = mbar_wait_warp(&st.mb[id], phase & 1u, &st.abort_flag);
+  ++phase;
+  return ok;
+}
+#define BAR_SYNC(id, count, phase) bar_sync_x(sh.bars, (id), (phase))
+#define BAR_ARRIVE(id, count) bar_arrive_x(sh.bars, (id))
+#define BAR_FAILED() (sh.bars.abort_flag != 0)
+#else
+__device__ __forceinline__ bool bar_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+  return true;
 }
 __device__ __forceinline__ void bar_arrive(int id, int count) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
+#define BAR_SYNC(id, count, phase) bar_sync((id), (count))
+#define BAR_ARRIVE(id, count) bar_arrive((id), (count))
+#define BAR_FAILED() false
+#endif
+
+struct WinShared {
+  StepMeta meta[2];
+  double u2[2];  // U(j, j+2), from the helper to the I/O warp
+  RowPk pk[2][32];
+#ifdef BANDLU_BOUNDED_SYNC
+  BarState bars;
+#endif
+};
+
+
+// Out of line, so that the rarely taken division is not if-converted into the
+// pivot chain of the panel warp.
+__device__ __noinline__ double div_slow(double x) { return 1.0 / x; }
 
 template <int K, int PF>
 __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, int ku, double *__restrict__ AB,
@@ -84,6 +138,9 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
   const int CS = kl + kv + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
+#ifdef BANDLU_BOUNDED_SYNC
+  if (threadIdx.x == 0) bar_init(sh.bars);
+#endif
   // Fill-row entries of the top-left corner (element row < 0) are cleared, as
   // the elimination clears every fill row before it starts.
   for (int e = threadIdx.x; e < kl * kv; e += blockDim.x) {
@@ -104,63 +161,92 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
 
   int info = 0;
   if (warp == 0) {
-    // ---------------- panel warp ----------------
+    // ---------------- panel warp: the pivot chain only ----------------
     int slot_reg = lane;  // slot of logical row j+lane (lanes < R)
     double cur = (lane <= kl && lane < n) ? W[lane * CS] : 0.0;
     int qn = 1 % CS;  // column slot of column j+1
+    unsigned ph_col = 0;
     for (int j = 0; j < n; ++j) {
       const int km = min(kl, n - 1 - j);
       const bool valid = lane <= km;
-      const unsigned long long key = valid ? abs_key(cur) : 0ull;
-      // Every candidate's reciprocal is formed (integer pipes) while the argmax runs.
-      const double rl = rcp_rn((valid && nz(cur)) ? cur : 1.5);
-      const int p = warp_argmax_first(key);
-      const double pv = __shfl_sync(FULL, cur, p);
-      const double r = __shfl_sync(FULL, rl, p);
-      const double c0 = __shfl_sync(FULL, cur, 0);
-      const bool zp = !nz(pv);  // exact zero pivot (then p == 0)
-      if (lane == p) cur = c0;
-      if (lane == 0) cur = pv;
-      const int s0 = __shfl_sync(FULL, slot_reg, 0);
-      const int sp = __shfl_sync(FULL, slot_reg, p);
-      if (lane == p) slot_reg = s0;
-      if (lane == 0) slot_reg = sp;
-      // column j+1, logical rows j .. j+kl+1 (holds steps <= j-1)
-      if (j >= 1) bar_sync(kBarCol, 64);
+      bool zp;  // exact zero pivot (then p == 0)
+      const int p = warp_argmax_first_z(valid ? abs_key(cur) : 0ull, &zp);
+      // interchange rows j and j+p: lanes 0 and p trade their values and slots
+      const int src = lane == 0 ? p : (lane == p ? 0 : lane);
+      slot_reg = __shfl_sync(FULL, slot_reg, src);
+      // column j+1, logical rows j .. j+kl+1 (holds steps <= j-1): the load is
+      // issued here and lands while the reciprocal is formed
+      if (j >= 1 && !BAR_SYNC(kBarCol, 64, ph_col)) break;
       double v = 0.0;
       if (j + 1 < n && lane <= kl + 1 && j + lane < n) v = W[slot_reg * CS + qn];
+      const double pv = __shfl_sync(FULL, cur, p);
+      bool rspec;
+      double r = rcp_rn_fast(zp ? 1.5 : pv, &rspec);  // integer pipes
+      if (rspec && !zp) r = div_slow(pv);               // subnormal / huge pivot: plain division
+      cur = __shfl_sync(FULL, cur, src);
       // U(j, j+1); when kv == 0 (diagonal matrix) column j+1 lies outside row j's band
       const double u = kv >= 1 ? __shfl_sync(FULL, v, 0) : 0.0;
       const double l = (!zp && lane >= 1 && valid) ? cur * r : cur;
-      // buffer b was last read in step j-2, which every updater finished before
-      // warp 1 reached kBarCol(j-1)
+      // step j on column j+1 before the updaters' multiply-adds start competing
+      // for the FP64 unit
+      if (j + 1 < n && !zp && nz(u) && lane >= 1 && valid) v = fma(-l, u, v);
+      // buffer b was last read in step j-2, which every reader finished before
+      // the helper reached kBarCol(j-1)
       const int b = j & 1;
       sh.pk[b][lane].l = l;
       sh.pk[b][lane].rb = slot_reg * CS;
-      if (lane == 0) sh.zp[b] = zp ? 1 : 0;
-      __syncwarp();
-      bar_arrive(kBarPub, kPubCount);
-      if (j + 1 < n) {
-        if (!zp && nz(u) && lane >= 1 && valid) v = fma(-l, u, v);
-        cur = __shfl_down_sync(FULL, v, 1);  // logical rows j+1 .. j+1+kl
-      }
       if (lane == 0) {
-        ipiv[j] = j + p + 1;
-        AB[kv + j * ldab] = pv;
-        if (kv >= 1 && j + 1 < n) AB[(kv - 1) + (j + 1) * ldab] = u;
+        sh.meta[b].u1 = u;
+        sh.meta[b].zp = zp ? 1 : 0;
+        sh.meta[b].p = p;
       }
-      if (lane >= 1 && valid) AB[(kv + lane) + j * ldab] = l;
+      __syncwarp();
+      BAR_ARRIVE(kBarPub, kPubCount);
+      cur = __shfl_down_sync(FULL, v, 1);  // logical rows j+1 .. j+1+kl
       if (zp && info == 0) info = j + 1;
-      const int sfirst = __shfl_sync(FULL, slot_reg, 0);
-      const int sn = __shfl_down_sync(FULL, slot_reg, 1);
-      slot_reg = (lane == R - 1) ? sfirst : sn;  // retired row's slot takes row j+R
+      // retired row j's slot takes row j+R
+      slot_reg = __shfl_sync(FULL, slot_reg, lane == R - 1 ? 0 : lane + 1);
       qn = (qn + 1 == CS) ? 0 : qn + 1;
     }
-    bar_sync(kBarCol, 64);  // warp 1's arrival of the last step
-  } else if (warp == kPrefetchWarp) {
-    // ---------------- row prefetch warp ----------------
-    // Row j-1+R enters the slot that row j-1 left; it is fetched in step j and
-    // stored in step j+1 (a whole step for the global loads to land).
+    if (!BAR_FAILED()) BAR_SYNC(kBarCol, 64, ph_col);  // the helper's arrival of the last step
+  } else if (warp == kHelperWarp) {
+    // ---------------- helper warp: column j+2 and the hand-off ----------------
+    int qj = 0;
+    unsigned ph_pub = 0;
+    for (int j = 0; j < n; ++j) {
+      const int b = j & 1;
+      if (!BAR_SYNC(kBarPub, kPubCount, ph_pub)) break;
+      const int km = min(kl, n - 1 - j);
+      const bool zp = sh.meta[b].zp != 0;
+      const int rb0 = sh.pk[b][0].rb;
+      if (j + 2 <= min(j + kv, n - 1)) {
+        int q = qj + 2;
+        if (q >= CS) q -= CS;
+        const double u = W[rb0 + q];
+        if (lane == 0) sh.u2[b] = u;  // U(j, j+2), written out by the I/O warp
+        if (!zp && nz(u) && lane >= 1 && lane <= km) {
+          const RowPk pk = sh.pk[b][lane];
+          W[pk.rb + q] = fma(-pk.l, u, W[pk.rb + q]);
+        }
+      }
+      // Column j+1+kv enters the window at step j+1.  Rows j+1..j+kl (any
+      // physical row pushed down by interchanges) hold structural zeros there;
+      // their slots may still hold a column that left the window CS steps ago.
+      if (lane >= 1 && lane <= kl && j + 1 + kv < n) {
+        int qe = qj + 1 + kv;
+        if (qe >= CS) qe -= CS;
+        W[sh.pk[b][lane].rb + qe] = 0.0;
+      }
+      __syncwarp();
+      BAR_ARRIVE(kBarCol, 64);
+      qj = (qj + 1 == CS) ? 0 : qj + 1;
+    }
+  } else if (warp == kIoWarp) {
+    // ---------------- I/O warp ----------------
+    // Step j's pivot, U diagonal, U(j, j+1), U(j, j+2) and multipliers go to
+    // global memory; then the row prefetch: row j-1+R enters the slot that row
+    // j-1 left; it is fetched in step j and stored in step j+1 (a whole step for
+    // the global loads to land).
     int pfo[PF];
 #pragma unroll
     for (int k = 0; k < PF; ++k) pfo[k] = (kDelta + lane + 32 * k) % CS;
@@ -168,9 +254,19 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
     bool have_pf = false;
     int pf_rb = 0, pf_q = 0;
     int qj = 0;
+    unsigned ph_pub = 0;
     for (int j = 0; j < n; ++j) {
       const int b = j & 1;
-      bar_sync(kBarPub, kPubCount);
+      if (!BAR_SYNC(kBarPub, kPubCount, ph_pub)) break;
+      const int km = min(kl, n - 1 - j);
+      // U(j, j+2) of the previous step: the helper wrote it before kBarPub(j)
+      if (lane == 0 && j >= 1 && kv >= 2 && j + 1 < n) AB[(kv - 2) + (long long)(j + 1) * ldab] = sh.u2[b ^ 1];
+      if (lane == 0) {
+        ipiv[j] = j + sh.meta[b].p + 1;
+        AB[kv + (long long)j * ldab] = sh.pk[b][0].l;
+        if (kv >= 1 && j + 1 < n) AB[(kv - 1) + (long long)(j + 1) * ldab] = sh.meta[b].u1;
+      }
+      if (lane >= 1 && lane <= km) AB[(kv + lane) + (long long)j * ldab] = sh.pk[b][lane].l;
       if (have_pf) {
 #pragma unroll
         for (int k = 0; k < PF; ++k) {
@@ -197,54 +293,34 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
       qj = (qj + 1 == CS) ? 0 : qj + 1;
     }
   } else if ((warp & 3) != 0) {
-    // ---------------- updater warps ----------------
-    const int uw = warp - 1 - (warp >> 2);  // 0..kNU-1
+    // ---------------- updater warps: columns j+3 .. j+kv ----------------
+    const int uw = warp - 1 - (warp >> 2) - (warp > kIoWarp ? 1 : 0);  // 0..kNU-1
     const int tid_u = uw * 32 + lane;
-    const int rows = kl + 1;
-    const int E = kv > 2 ? (kv - 2) * rows : 0;
-    // Static element map of columns j+3..j+kv: element e -> column offset
-    // d = 3 + e / rows, row offset t = e % rows (t = 0: the U row is written out).
+    const int ncols = kv > 2 ? kv - 2 : 0;
+    const int E = ncols * (kl + 1);
+    // Static element map, columns fastest: element e -> row offset t = e / ncols
+    // (t = 0: the U row is written out), column offset d = 3 + e % ncols.  The
+    // lanes of a warp then read one row record (a broadcast) and consecutive
+    // columns of the pivot row and of their own row (no bank conflicts).
     int ed[K], et[K];
     long long uoff[K];  // offset of U(j, j+d) in AB relative to column j
 #pragma unroll
     for (int k = 0; k < K; ++k) {
       const int e = tid_u + kNUT * k;
-      ed[k] = e < E ? 3 + e / rows : 0;
-      et[k] = e < E ? e - (ed[k] - 3) * rows : 0;
+      et[k] = e < E ? e / ncols : 0;
+      ed[k] = e < E ? 3 + (e - et[k] * ncols) : 0;
       uoff[k] = (kv - ed[k]) + (long long)ed[k] * ldab;
     }
     int qj = 0;  // column slot of column j
+    unsigned ph_pub = 0;
     for (int j = 0; j < n; ++j) {
       const int b = j & 1;
-      bar_sync(kBarPub, kPubCount);
+      if (!BAR_SYNC(kBarPub, kPubCount, ph_pub)) break;
       const int km = min(kl, n - 1 - j);
-      const bool zp = sh.zp[b] != 0;
+      const bool zp = sh.meta[b].zp != 0;
       const int cmax = min(j + kv, n - 1);
       const int rb0 = sh.pk[b][0].rb;
-      if (warp == 1) {
-        const int c = j + 2;
-        if (c <= cmax) {
-          int q = qj + 2;
-          if (q >= CS) q -= CS;
-          const double u = W[rb0 + q];
-          if (lane == 0) AB[(kv - 2) + (long long)c * ldab] = u;
-          if (!zp && nz(u) && lane >= 1 && lane <= km) {
-            const RowPk pk = sh.pk[b][lane];
-            W[pk.rb + q] = fma(-pk.l, u, W[pk.rb + q]);
-          }
-        }
-        // Column j+1+kv enters the window at step j+1.  Rows j+1..j+kl (any
-        // physical row pushed down by interchanges) hold structural zeros there;
-        // their slots may still hold a column that left the window CS steps ago.
-        if (lane >= 1 && lane <= kl && j + 1 + kv < n) {
-          int qe = qj + 1 + kv;
-          if (qe >= CS) qe -= CS;
-          W[sh.pk[b][lane].rb + qe] = 0.0;
-        }
-        __syncwarp();
-        bar_arrive(kBarCol, 64);
-      }
-      // columns j+3..j+kv: all loads first, then the fused multiply-adds, then the stores
+      // all loads first, then the fused multiply-adds, then the stores
       const bool full = j + kv <= n - 1;  // every mapped element is inside the matrix
       double *ABj = AB + (long long)j * ldab;
       double uu[K], xx[K], ll[K];
@@ -276,7 +352,7 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
     }
   }
   __syncthreads();
-  if (threadIdx.x == 0) *d_info = info;
+  if (threadIdx.x == 0) *d_info = BAR_FAILED() ? -BANDLU_ERR_TIMEOUT : info;
 }
 
 __global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int ku, double *__restrict__ AB,

@@ -62,14 +62,17 @@ __host__ __device__ __forceinline__ uint32_t fbits(float x) {
 #endif
 }
 
-// Correctly rounded 1/b (IEEE binary64, round to nearest even).
-__host__ __device__ __forceinline__ double rcp_rn(double b) {
+// Correctly rounded 1/b for every b whose reciprocal is a normal number and
+// whose significand is not a power of two: *special is set for zeros,
+// subnormals, infinities, NaN and |b| >= 2^1021, and the value returned then is
+// meaningless.  Straight-line code (no branches), so it interleaves with other
+// work.
+__host__ __device__ __forceinline__ double rcp_rn_fast(double b, bool *special) {
   const uint64_t bits = dbits(b);
   const uint64_t E = (bits >> 52) & 0x7ffull;
   const uint64_t frac = bits & ((1ull << 52) - 1);
   const uint64_t sign = bits & (1ull << 63);
-  if (E == 0 || E >= 2045) return 1.0 / b;
-  if (frac == 0) return bitsd(sign | ((2046 - E) << 52));  // power of two: exact
+  *special = (E == 0) | (E >= 2045);
   const uint64_t m = frac | (1ull << 52);
   // M = m / 2^29 = xh + xl/2^29 with xh the 24-bit rounding (exact in single
   // precision) and |xl| <= 2^28.
@@ -91,15 +94,20 @@ __host__ __device__ __forceinline__ double rcp_rn(double b) {
   Q = (uint64_t)((int64_t)Q + (int64_t)(int32_t)((float)(int32_t)(R >> 31) * y * 4.0f));
   // now |Q - 2^105/m| < 1.01: the exact remainder fixes Q and decides the rounding
   R = (int64_t)(0ull - Q * m);
-  if (R < 0) {
-    Q -= 1;
-    R += (int64_t)m;
-  } else if (R >= (int64_t)m) {
-    Q += 1;
-    R -= (int64_t)m;
-  }
-  if ((uint64_t)R > m - (uint64_t)R) Q += 1;  // 2R > m: round up
-  return bitsd(sign | ((2045 - E) << 52) | (Q - (1ull << 52)));
+  const bool lo = R < 0, hi = R >= (int64_t)m;
+  Q = lo ? Q - 1 : (hi ? Q + 1 : Q);
+  R = lo ? R + (int64_t)m : (hi ? R - (int64_t)m : R);
+  Q += ((uint64_t)R > m - (uint64_t)R) ? 1ull : 0ull;  // 2R > m: round up
+  const uint64_t rbits = sign | ((2045 - E) << 52) | (Q - (1ull << 52));
+  const uint64_t pbits = sign | ((2046 - E) << 52);  // significand 1: 1/b is a power of two
+  return bitsd(frac == 0 ? pbits : rbits);
+}
+
+// Correctly rounded 1/b (IEEE binary64, round to nearest even).
+__host__ __device__ __forceinline__ double rcp_rn(double b) {
+  bool special;
+  const double r = rcp_rn_fast(b, &special);
+  return special ? 1.0 / b : r;
 }
 
 }  // namespace bandlu
