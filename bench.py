@@ -348,6 +348,103 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_workload_report(args):
+    """One JSON line per call for any workload (per-stage CUDA-event timings), used for the
+    per-workload table; the contract line is the default workload's."""
+    import torch
+
+    from paper_2608_22099_gb300 import bandlu
+    from paper_2608_22099_gb300.workloads import WORKLOADS, make_workload
+
+    w = WORKLOADS[args.workload]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    bandlu.load()
+    A = make_workload(w, device=dev)
+    n, kl, ku, ldab = w.n, w.kl, w.ku, w.ldab
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+    hbm_peak, hbm_src = load_peaks()
+    out = {"workload": w.name, "n": n, "kl": kl, "ku": ku, "batch": w.batch}
+    reps = max(1, args.steps)
+
+    def timed(fn, reps):
+        ts = []
+        for r in range(reps):
+            flush.fill_(r)
+            a = torch.cuda.Event(enable_timing=True); b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b) * 1e-3)
+        return statistics.median(ts)
+
+    if w.batch:
+        B = w.batch
+        AB = torch.zeros((B, n, ldab), dtype=torch.float64, device=dev)
+        ipiv = torch.zeros((B, n), dtype=torch.int32, device=dev)
+        kls, kus, infos, sts = (torch.zeros(B, dtype=torch.int32, device=dev) for _ in range(4))
+
+        def step():
+            bandlu.check(bandlu.dispatch_lu_batched(A, n, n, n * n, B, AB, ldab, n * ldab, ipiv, n, kls, kus,
+                                                    infos, sts, stream), "dispatch_lu_batched")
+        for _ in range(max(args.warmup, 3)):
+            step()
+        t = timed(step, reps)
+        diag = AB[:, :, kl + ku].cpu().numpy()
+        ip = ipiv.cpu().numpy()
+        flops = sum(band_flops(ip[b], diag[b], n, kl, ku) for b in range(B))
+        bytes_ = 8.0 * B * n * n
+        out.update({"dispatch_batched_ms": t * 1e3, "gflops": flops / t / 1e9, "hbm_gbs": bytes_ / t / 1e9,
+                    "hbm_frac": bytes_ / t / 1e9 / hbm_peak, "matrices_per_s": B / t, "flops": flops})
+    else:
+        AB = torch.zeros((n, ldab), dtype=torch.float64, device=dev)
+        ipiv = torch.zeros(n, dtype=torch.int32, device=dev)
+        info = torch.zeros(1, dtype=torch.int32, device=dev)
+        klku = torch.zeros(2, dtype=torch.int32, device=dev)
+        res = {}
+
+        def disp():
+            res["rc"] = bandlu.dispatch_lu(A, n, n, AB, ldab, ipiv, info, stream)
+
+        def det():
+            bandlu.check(bandlu.detect_bandwidth(A, n, n, klku, klku.data_ptr() + 4, stream), "detect")
+
+        for _ in range(max(args.warmup, 3)):
+            disp()
+        t_disp = timed(disp, reps)
+        t_det = timed(det, reps)
+        rc, dkl, dku = res["rc"]
+        out.update({"status": rc, "detected_kl": dkl, "detected_ku": dku, "dispatch_ms": t_disp * 1e3,
+                    "detect_us": t_det * 1e6, "detect_gbs": 8.0 * n * n / t_det / 1e9,
+                    "detect_frac_hbm": 8.0 * n * n / t_det / 1e9 / hbm_peak})
+        if rc == 0:
+            def conv():
+                bandlu.check(bandlu.dense_to_band(A, n, n, kl, ku, AB, ldab, stream), "convert")
+
+            AB2 = torch.zeros_like(AB)
+
+            def fac():
+                AB2.copy_(AB)
+                bandlu.check(bandlu.gbtrf(n, kl, ku, AB2, ldab, ipiv, info, stream), "gbtrf")
+            conv()
+            t_conv = timed(conv, reps)
+            t_fac = timed(fac, max(1, min(reps, 5))) if n > 20000 else timed(fac, reps)
+            flops = band_flops(ipiv.cpu().numpy(), AB2[:, kl + ku].cpu().numpy(), n, kl, ku)
+            out.update({"convert_us": t_conv * 1e6, "gbtrf_ms": t_fac * 1e3, "gbtrf_gflops": flops / t_fac / 1e9,
+                        "gbtrf_ns_per_column": t_fac / n * 1e9, "flops": flops,
+                        "gflops_dispatch": flops / t_disp / 1e9})
+        if n <= 20000:
+            Ac = A.clone()
+            t_dense = timed(lambda: torch.linalg.lu_factor(Ac.clone()), 3)
+            out["dense_lu_ms"] = t_dense * 1e3
+            out["speedup_over_dense" if rc == 0 else "slowdown_vs_dense"] = (
+                t_dense / t_disp if rc == 0 else (t_det + t_dense) / t_dense)
+    out["hbm_peak_source"] = hbm_src
+    print(json.dumps(out), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -355,9 +452,13 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="workload name (default: the n=4096, kl=ku=16 matrix); others for per-workload reports")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload != WORKLOAD:
+        run_workload_report(args)
     else:
         run_ours(args)
 
