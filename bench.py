@@ -15,6 +15,7 @@ data-parallel split), one per GPU.
 from __future__ import annotations
 
 import argparse
+import atexit
 import json
 import os
 import statistics
@@ -109,6 +110,27 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(inside)}
 
 
+def dense_lu_ms(torch, A, stream, reps: int = 3):
+    """Median time of the generic dense LU (the comparison F(N) of Sec. III-A, cuSOLVER getrf via
+    torch) on a copy of A, or None when torch's linear-algebra library is unavailable."""
+    times = []
+    try:
+        for _ in range(reps):
+            Ac = A.clone()
+            torch.cuda.synchronize()
+            a0 = torch.cuda.Event(enable_timing=True)
+            a1 = torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            torch.linalg.lu_factor(Ac)
+            a1.record(stream)
+            torch.cuda.synchronize()
+            times.append(a0.elapsed_time(a1))
+            del Ac
+    except RuntimeError:
+        return None
+    return statistics.median(times)
+
+
 def cpu_oracle_dispatch(A_np: np.ndarray, ldab: int, budget_s: float, max_steps: int):
     """Time the CPU oracle's dispatch (detect + decide + convert + banded LU) on the
     whole matrix, repeated while the time budget lasts."""
@@ -198,6 +220,7 @@ def run_ours(args):
     sampler = ClockSampler(local)
     if rank == 0:
         sampler.start()
+        atexit.register(sampler.stop)  # never leave the sampler running if the bench fails
         time.sleep(0.3)
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
@@ -300,18 +323,7 @@ def run_ours(args):
     d2h = AB_host.numel() * 8 + ipiv_host.numel() * 4 + info_host.numel() * 4
 
     # the generic algorithm F(N) of Sec. III-A on the same matrix: dense LU (cuSOLVER via torch)
-    dense_ms = []
-    for _ in range(3):
-        Ac = A.clone()
-        torch.cuda.synchronize()
-        a0 = torch.cuda.Event(enable_timing=True); a1 = torch.cuda.Event(enable_timing=True)
-        a0.record(stream)
-        torch.linalg.lu_factor(Ac)
-        a1.record(stream)
-        torch.cuda.synchronize()
-        dense_ms.append(a0.elapsed_time(a1))
-        del Ac
-    dense_t = statistics.median(dense_ms)
+    dense_t = dense_lu_ms(torch, A, stream)
 
     clocks = None
     if rank == 0:
@@ -334,7 +346,8 @@ def run_ours(args):
             "config": {"workload": WORKLOAD, "n": n, "kl": kl, "ku": ku, "ldab": ldab, "dist": "uniform[-1,1]",
                        "l2": "flushed between steps (512 MiB write)",
                        "parallelism": "replicas" if world > 1 else "single"},
-            "dispatch_ms": ms_per_step, "speedup_over_dense": dense_t / ms_per_step, "dense_lu_ms": dense_t,
+            "dispatch_ms": ms_per_step, "dense_lu_ms": dense_t,
+            "speedup_over_dense": (dense_t / ms_per_step) if dense_t else None,
             "flops_per_step": flops, "stages": stages, "roofline": roofline,
             "cpu_baseline": cpu_baseline,
             "e2e": {"value": e2e_value, "unit": "GFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -436,11 +449,12 @@ def run_workload_report(args):
                         "gbtrf_ns_per_column": t_fac / n * 1e9, "flops": flops,
                         "gflops_dispatch": flops / t_disp / 1e9})
         if n <= 20000:
-            Ac = A.clone()
-            t_dense = timed(lambda: torch.linalg.lu_factor(Ac.clone()), 3)
-            out["dense_lu_ms"] = t_dense * 1e3
-            out["speedup_over_dense" if rc == 0 else "slowdown_vs_dense"] = (
-                t_dense / t_disp if rc == 0 else (t_det + t_dense) / t_dense)
+            d_ms = dense_lu_ms(torch, A, stream)
+            out["dense_lu_ms"] = d_ms
+            if d_ms:
+                t_dense = d_ms * 1e-3
+                out["speedup_over_dense" if rc == 0 else "slowdown_vs_dense"] = (
+                    t_dense / t_disp if rc == 0 else (t_det + t_dense) / t_dense)
     out["hbm_peak_source"] = hbm_src
     print(json.dumps(out), flush=True)
 

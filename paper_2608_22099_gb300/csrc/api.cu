@@ -86,7 +86,7 @@ int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA
   if (strideA < n * lda) return -4;
   if (batch < 0) return -5;
   if (AB == nullptr && work) return -6;
-  if (ldab < 1) return -7;
+  if (ldab < 1 || ldab > (int64_t)INT_MAX) return -7;
   if (strideAB < n * ldab) return -8;
   if (ipiv == nullptr && work) return -9;
   if (strideP < n) return -10;

@@ -109,58 +109,65 @@ __global__ void __launch_bounds__(256) k_batch_scan_convert(const double *__rest
 }
 
 // Unblocked banded elimination by one warp on band storage `ab` (shared or
-// global memory).  Returns info.
-__device__ int warp_gbtrf(double *ab, long long ldab, long long n, int kl, int ku, int *ipiv) {
+// global memory), in the xGBTRF order of operations.  32-bit indices (n < 2^31).
+// Candidates of a pivot column sit one per lane; the first-max argmax is the
+// exact integer reduction over |x|'s bit pattern.  Returns info.
+__device__ int warp_gbtrf(double *ab, int ldab, int n, int kl, int ku, int *ipiv) {
   const int lane = threadIdx.x & 31;
-  const long long kv = (long long)kl + ku;
+  const int kv = kl + ku;
   if (kl > 0) {
-    for (long long e = lane; e < n * kl; e += 32) {
+    for (long long e = lane; e < (long long)n * kl; e += 32) {
       const long long c = e / kl, r = e - c * kl;
       ab[r + c * ldab] = 0.0;
     }
   }
   __syncwarp();
-  long long ju = 0;
+  int ju = 0;
   int info = 0;
-  for (long long j = 0; j < n; ++j) {
-    const long long km = min((long long)kl, n - 1 - j);
-    double *col = ab + j * ldab;
-    KeyIdx best{0ull, LLONG_MAX};
-    for (long long t = lane; t <= km; t += 32) best = better(best, KeyIdx{abs_key(col[kv + t]), t});
-    best = warp_reduce_keyidx(best);
-    const long long p = best.idx;
+  for (int j = 0; j < n; ++j) {
+    const int km = min(kl, n - 1 - j);
+    double *col = ab + (long long)j * ldab;
+    int p;
+    if (km < 32) {
+      const double x = lane <= km ? col[kv + lane] : 0.0;
+      bool allz;
+      p = warp_argmax_first_z(lane <= km ? abs_key(x) : 0ull, &allz);
+    } else {
+      KeyIdx best{0ull, LLONG_MAX};
+      for (int t = lane; t <= km; t += 32) best = better(best, KeyIdx{abs_key(col[kv + t]), t});
+      p = (int)warp_reduce_keyidx(best).idx;
+    }
     const double pv = col[kv + p];
-    if (lane == 0) ipiv[j] = (int)(j + p + 1);
-    __syncwarp();
+    if (lane == 0) ipiv[j] = j + p + 1;
     if (nz(pv)) {
       ju = max(ju, min(j + ku + p, n - 1));
       if (p != 0) {
-        for (long long c = j + lane; c <= ju; c += 32) {
-          double *x = ab + (kv + j - c) + c * ldab;
-          double *y = ab + (kv + j + p - c) + c * ldab;
+        for (int c = j + lane; c <= ju; c += 32) {
+          double *x = ab + (kv + j - c) + (long long)c * ldab;
+          double *y = ab + (kv + j + p - c) + (long long)c * ldab;
           const double t0 = *x;
           *x = *y;
           *y = t0;
         }
-        __syncwarp();
       }
       if (km > 0) {
         const double r = rcp_rn(pv);  // IEEE 1/pv on the integer pipes
-        for (long long t = 1 + lane; t <= km; t += 32) col[kv + t] *= r;
         __syncwarp();
-        const long long tot = (ju - j) * km;
-        for (long long e = lane; e < tot; e += 32) {
-          const long long cc = e / km, t = 1 + (e - cc * km);
-          const long long c = j + 1 + cc;
-          double *colc = ab + c * ldab;
+        for (int t = 1 + lane; t <= km; t += 32) col[kv + t] *= r;
+        __syncwarp();
+        const int ncol = ju - j;
+        for (int e = lane; e < ncol * km; e += 32) {
+          const int cc = e / km, t = 1 + (e - cc * km);
+          const int c = j + 1 + cc;
+          double *colc = ab + (long long)c * ldab;
           const double u = colc[kv + j - c];
           if (nz(u)) colc[kv + j + t - c] = fma(-col[kv + t], u, colc[kv + j + t - c]);
         }
-        __syncwarp();
       }
     } else if (info == 0) {
-      info = (int)(j + 1);
+      info = j + 1;
     }
+    __syncwarp();
   }
   return info;
 }
@@ -183,11 +190,11 @@ __global__ void __launch_bounds__(128) k_batch_factor(long long n, long long bat
     const long long total = n * ldab;
     for (long long e = lane; e < total; e += 32) s[e] = ABb[e];
     __syncwarp();
-    info = warp_gbtrf(s, ldab, n, kl, ku, ipiv + b * strideP);
+    info = warp_gbtrf(s, (int)ldab, (int)n, kl, ku, ipiv + b * strideP);
     __syncwarp();
     for (long long e = lane; e < total; e += 32) ABb[e] = s[e];
   } else {
-    info = warp_gbtrf(ABb, ldab, n, kl, ku, ipiv + b * strideP);
+    info = warp_gbtrf(ABb, (int)ldab, (int)n, kl, ku, ipiv + b * strideP);
   }
   if (lane == 0) d_info[b] = info;
 }
