@@ -85,7 +85,13 @@ namespace bandlu {
 int launch_detect(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t s);
 int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
                          cudaStream_t s);
-int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s);
+// allow_alloc = false keeps the launch free of device allocations (wide bands
+// then take the single-CTA kernel instead of the multi-CTA one, whose
+// hand-off flags live in stream-ordered scratch).
+int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s,
+                 bool allow_alloc = true);
+int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s,
+                      bool *used);
 int launch_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,
                    int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku, int *d_info,
                    int *d_status, cudaStream_t s);

@@ -1,6 +1,7 @@
 // gbtrf.cu -- banded LU with partial pivoting (Sec. II-A step 3; f(N) ~ O(N*P*Q), Eq. S-N-N3).
 //
-// Two single-matrix kernels:
+// Two single-matrix kernels here (wide bands go first to the multi-CTA kernel
+// of gbtrf_wide.cu, when it can be launched):
 //
 //  * k_gbtrf_window (kl <= 27, the narrow bands the method targets).  One CTA.
 //    The active part of the band at step j is the dense (kl+1) x (kv+1) block
@@ -450,7 +451,8 @@ int launch_window_pf(int pf, long long n, int kl, int ku, double *AB, long long 
 
 }  // namespace
 
-int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s) {
+int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s,
+                 bool allow_alloc) {
   if (n == 0) {
     if (cudaMemsetAsync(d_info, 0, sizeof(int), s) != cudaSuccess) return BANDLU_ERR_CUDA;
     return BANDLU_OK;
@@ -467,6 +469,11 @@ int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv,
     if (k <= 2) return launch_window_pf<2>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
     if (k <= 4) return launch_window_pf<4>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
     return launch_window_pf<8>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+  }
+  if (allow_alloc) {
+    bool used = false;
+    const int rc = launch_gbtrf_wide(n, kl, ku, AB, ldab, ipiv, d_info, s, &used);
+    if (rc != BANDLU_OK || used) return rc;
   }
   k_gbtrf_generic<<<1, 1024, 0, s>>>(n, kl, ku, AB, ldab, ipiv, d_info);
   BANDLU_CHECK_LAUNCH();

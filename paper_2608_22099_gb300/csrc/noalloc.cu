@@ -73,5 +73,5 @@ extern "C" int dispatch_lu_noalloc(const double *A, int64_t n, int64_t lda, doub
   if (!bandlu::predicate_banded(n, h[0], h[1], ldab)) return BANDLU_NOT_BANDED;
   rc = bandlu::launch_dense_to_band(A, lda, n, h[0], h[1], AB, ldab, stream);
   if (rc != BANDLU_OK) return rc;
-  return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream);
+  return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream, /*allow_alloc=*/false);
 }

@@ -203,6 +203,51 @@ def test_gbtrf_empty():
 
 
 # --------------------------------------------------------------------------------------------
+# wide bands (kl beyond the windowed kernel): the multi-CTA panel/update kernel
+# --------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,kl,ku", [(12, 28, 0), (13, 29, 1), (50, 30, 28), (203, 28, 0), (401, 33, 70),
+                                     (777, 64, 5), (1030, 100, 100), (2049, 256, 256)])
+def test_gbtrf_wide_matches_oracle(n, kl, ku):
+    A = banded(n, kl, ku, seed=11 * n + kl + 3 * ku, dist="normal").numpy()
+    AB = oracle.dense_to_band(A, kl, ku)
+    ref = oracle.gbtrf(AB, kl, ku)
+    got = gbtrf_gpu(AB, kl, ku)
+    assert_factor_parity(*got, ref[0], ref[1], ref[2])
+    assert oracle.backward_error(A, got[0], got[1], kl, ku) <= 10.0
+
+
+def test_gbtrf_wide_blocks_share_update_ctas():
+    # kv = 700: one panel reaches more column blocks than there are update CTAs,
+    # so update CTAs hold two blocks at once.
+    n, kl, ku = 2003, 300, 400
+    A = banded(n, kl, ku, seed=17, boost=2.0).numpy()
+    AB = oracle.dense_to_band(A, kl, ku)
+    ref = oracle.gbtrf(AB, kl, ku)
+    assert_factor_parity(*gbtrf_gpu(AB, kl, ku), ref[0], ref[1], ref[2])
+
+
+def test_gbtrf_wide_zero_pivots_garbage_fill_and_wider_storage():
+    n, kl, ku = 500, 40, 31
+    A = banded(n, kl, ku, seed=23).numpy()
+    A[:, 77] = 0.0
+    A[200:240, 200:240] = 0.0
+    AB = oracle.dense_to_band(A, kl, ku, ldab=2 * kl + ku + 1 + 5)
+    AB[:, :kl] = -9.5
+    ref = oracle.gbtrf(AB, kl, ku)
+    assert ref[2] > 0
+    assert_factor_parity(*gbtrf_gpu(AB, kl, ku), ref[0], ref[1], ref[2])
+
+
+def test_gbtrf_wide_deterministic():
+    n, kl, ku = 1500, 48, 48
+    AB = oracle.dense_to_band(banded(n, kl, ku, seed=2).numpy(), kl, ku)
+    a = gbtrf_gpu(AB, kl, ku)
+    b = gbtrf_gpu(AB, kl, ku)
+    assert np.array_equal(a[0].view(np.int64), b[0].view(np.int64)) and np.array_equal(a[1], b[1])
+
+
+# --------------------------------------------------------------------------------------------
 # dispatch_lu and dispatch_lu_batched
 # --------------------------------------------------------------------------------------------
 

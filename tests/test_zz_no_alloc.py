@@ -44,3 +44,14 @@ def test_noalloc_declines_like_dispatch_lu():
     got = run(bandlu.dispatch_lu_noalloc, Ad, 10)
     assert got[:3] == ref[:3] == (bandlu.BANDLU_NOT_BANDED, 999, 3)
     assert np.all(got[3] == -3.0) and np.all(got[4] == -1) and got[5] == -5
+
+
+def test_noalloc_wide_band_matches_dispatch_lu():
+    # wide band: dispatch_lu takes the multi-CTA kernel, the allocation-free entry
+    # point the single-CTA one; both reproduce the unblocked elimination exactly
+    A = make_dense(1200, 40, 30, dist="normal", seed=91)
+    Ad = A.to(DEV)
+    ref = run(bandlu.dispatch_lu, Ad, 111)
+    got = run(bandlu.dispatch_lu_noalloc, Ad, 111)
+    assert got[:3] == ref[:3] == (0, 40, 30)
+    assert_factor_parity(got[3], got[4], got[5], ref[3], ref[4], ref[5])
