@@ -14,7 +14,12 @@ constexpr unsigned FULL = 0xffffffffu;
 // (NaN, +-Inf and subnormals are nonzero).  Integer-only, so it never issues on
 // the FP64 pipe.
 __device__ __forceinline__ bool nz_bits(unsigned long long b) { return (b << 1) != 0ull; }
-__device__ __forceinline__ bool nz(double x) { return nz_bits((unsigned long long)__double_as_longlong(x)); }
+// The same test on a double, done on its two 32-bit halves: the 64-bit form of
+// a double's bits can be compiled back into a floating-point compare, which
+// issues on the FP64 pipe at the FMA rate.
+__device__ __forceinline__ bool nz(double x) {
+  return ((((unsigned)__double2hiint(x)) << 1) | (unsigned)__double2loint(x)) != 0u;
+}
 
 // |x| as an unsigned key: for non-NaN doubles, |x| < |y| iff key(x) < key(y).
 __device__ __forceinline__ unsigned long long abs_key(double x) {

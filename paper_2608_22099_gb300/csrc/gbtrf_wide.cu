@@ -2,85 +2,115 @@
 // a persistent, cooperatively launched kernel, one CTA per SM (Sec. II-A step 3;
 // f(N) ~ O(N*P*Q), Eq. S-N-N3).
 //
-// The columns are cut into blocks of kNB.  Block p is panel p.
-//  * CTA 0 (panel CTA) factors panel p in shared memory (unblocked, the xGBTRF
-//    order of operations), writes it to AB and publishes it (panel_ready[p]);
-//    then it applies panel p to block p+1 (one-panel lookahead), which thereby
-//    becomes panel p+1, fully updated.
-//  * CTAs 1..G-1 (update CTAs) own the blocks b >= 2, block b on CTA
-//    1 + (b-2) mod (G-1).  A block is read into shared memory when the first
-//    panel reaching it is published, receives panels p_first(b)..b-2 in order,
-//    and is handed to the panel CTA (written to AB, block_ready[b]) one panel
-//    before the panel CTA needs it.
-// Every entry receives exactly the fma sequence of the unblocked elimination,
-// in the same order (the interchanges are the same permutations applied to
-// the same values), so the factors are bit-identical to it.
+// Columns are cut into blocks of kNB; block p is panel p.
 //
-// Hand-offs are acquire/release flags in global memory with bounded waits: a
-// wait that gives up raises an error flag that every CTA checks, the kernel
-// ends, and *d_info becomes -BANDLU_ERR_TIMEOUT.
+//  * CTA 0 (panel CTA).  Nine compute warps own the rows of the current panel
+//    (thread i <-> row p*kNB + i, held in registers).  One panel step is one
+//    exact argmax round and ONE barrier: every warp publishes its best
+//    candidate together with that row's panel values, and the thread of row j
+//    publishes row j, so every thread can apply the interchange, form its
+//    multiplier and update its own row without further synchronisation.
+//    After panel p the compute warps apply panel p-1 and panel p to block p+1
+//    (a two-panel lookahead), which thereby becomes panel p+1.
+//    An I/O warp writes every finished panel block and its pivots to AB and
+//    ipiv, publishes them (panel_ready[p]), and prefetches block p+2 with
+//    cp.async once its owner has handed it over (block_ready[p+2]).
+//  * CTAs 1..G (update CTAs) own the blocks b >= 3, block b on CTA
+//    1 + (b-3) mod G.  A block is read into shared memory when the first panel
+//    reaching it is published, receives panels p_first(b)..b-3 in order, and is
+//    handed to the panel CTA (written to AB, block_ready[b]) two panels before
+//    the panel CTA needs it.
+//
+// Every entry receives exactly the fma sequence of the unblocked elimination
+// in the same order (the interchanges permute the same values, the multiplier
+// is the pivot's correctly rounded reciprocal times the entry, each update is
+// fma(-l, u, a) with the zero-u skip), so the factors are bit-identical to it.
+// Interchanges and updates are applied up to the band's reach j + kv instead
+// of the running column reach ju: beyond ju both interchanged entries and the
+// row-j entry are +0.0 fill, so this changes no bit.
+//
+// Hand-offs between CTAs are acquire/release flags in global memory, inside
+// the panel CTA mbarriers; every wait is bounded.  A wait that gives up raises
+// an error flag that every waiter checks, the kernel ends, and *d_info becomes
+// -BANDLU_ERR_TIMEOUT.
 #include <climits>
+#include <cstdint>
 
 #include "common.cuh"
 #include "rcp.cuh"
+#include "sync.cuh"
 
 namespace bandlu {
 namespace {
 
-constexpr int kNB = 4;          // panel width = column block width
-constexpr int kThreads = 256;
-constexpr int kMaxActive = 2;   // blocks an update CTA holds at once
-constexpr long long kSpinLimitCycles = 2000000000ll;
+constexpr int kNB = 4;                // panel width = column block width
+constexpr int kCW = 9;                // compute warps
+constexpr int kCT = 32 * kCW;         // compute threads
+constexpr int kThreads = kCT + 32;    // + the panel CTA's I/O warp
+constexpr int kMaxActive = 2;         // blocks an update CTA holds at once
+constexpr int kPanelBufs = 3;         // block buffers of the panel CTA
+constexpr long long kSpinLimit = 2000000000ll;
+
+__device__ __forceinline__ void bar_compute() { asm volatile("bar.sync 1, %0;" ::"n"(kCT) : "memory"); }
 
 __device__ __forceinline__ int ld_acquire(const int *p) {
   int v;
   asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
+__device__ __forceinline__ int ld_relaxed(const int *p) {
+  int v;
+  asm volatile("ld.relaxed.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
 __device__ __forceinline__ void st_release(int *p, int v) {
   asm volatile("st.release.gpu.global.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
-// Whole CTA: thread 0 waits for *flag != 0 (bounded), the result is shared.
-__device__ bool cta_wait(const int *flag, int *err, int *s_ok) {
-  if (threadIdx.x == 0) {
-    int ok = 1;
-    const long long t0 = clock64();
-    for (unsigned it = 0;; ++it) {
-      if (ld_acquire(flag) != 0) break;
-      if (ld_acquire(err) != 0) {
-        ok = 0;
-        break;
-      }
-      if ((it & 63u) == 63u && clock64() - t0 > kSpinLimitCycles) {
-        atomicExch(err, 1);
-        ok = 0;
-        break;
-      }
-      __nanosleep(64);
-    }
-    *s_ok = ok;
-  }
-  __syncthreads();
-  const bool ok = *s_ok != 0;
-  __syncthreads();
-  return ok;
+// Pivot-search key of a candidate, so that the FIRST largest key is the row
+// the xGBTRF comparison order picks: the running best starts at the first
+// candidate and a later one replaces it only if strictly larger in modulus.
+// NaN never compares larger, so it wins only as the first candidate.  Keys are
+// offset by one so that 0 means "not a candidate".
+__device__ __forceinline__ unsigned long long pivot_key(double a, bool first) {
+  const unsigned hi = (unsigned)__double2hiint(a) & 0x7fffffffu, lo = (unsigned)__double2loint(a);
+  const bool nan = hi > 0x7ff00000u || (hi == 0x7ff00000u && lo != 0u);
+  const unsigned long long b = ((unsigned long long)hi << 32) | lo;
+  return nan ? (first ? 0x8000000000000000ull : 1ull) : b + 1ull;
 }
 
-// Whole CTA: make this CTA's global writes visible, then set *flag.
-__device__ void cta_signal(int *flag) {
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) st_release(flag, 1);
+// First lane holding the largest key; *kmax receives that key.
+__device__ __forceinline__ int warp_first_max(unsigned long long key, unsigned long long *kmax) {
+  const unsigned hi = (unsigned)(key >> 32), lo = (unsigned)key;
+  const unsigned mhi = __reduce_max_sync(FULL, hi);
+  const unsigned mlo = __reduce_max_sync(FULL, hi == mhi ? lo : 0u);
+  *kmax = ((unsigned long long)mhi << 32) | mlo;
+  return __ffs(__ballot_sync(FULL, hi == mhi && lo == mlo)) - 1;
+}
+
+// Bit d set iff u[d] != 0.0.
+__device__ __forceinline__ unsigned nz_mask(const double (&u)[kNB]) {
+  unsigned m = 0;
+#pragma unroll
+  for (int d = 0; d < kNB; ++d) m |= nz(u[d]) ? (1u << d) : 0u;
+  return m;
+}
+// One elimination update a - l*u with the zero-u skip (unz = u != 0), branch
+// free: the fma is always issued and its result discarded when u is +-0 (so a
+// signed zero a and an infinite l stay as the skip leaves them).
+__device__ __forceinline__ double upd(double l, double u, double a, bool unz) {
+  const double t = fma(-l, u, a);
+  return unz ? t : a;
 }
 
 struct Geo {
   int n, kl, ku, kv;
   long long ldab;
   int npan;
+  bool vec;  // AB is 16-byte aligned: blocks move as 16-byte chunks
 };
 
-// First panel whose U rows reach block b: panel p reaches column (p+1)*kNB - 1 + kv.
+// First panel whose U rows reach block b (panel p reaches column (p+1)*kNB - 1 + kv).
 __device__ __forceinline__ int p_first(const Geo &g, int b) {
   const int x = b * kNB - g.kv + 1;
   return x <= 0 ? 0 : (x + kNB - 1) / kNB - 1;
@@ -89,254 +119,518 @@ __device__ __forceinline__ int p_first(const Geo &g, int b) {
 __device__ __forceinline__ int b_last(const Geo &g, int p) {
   return min(g.npan - 1, ((p + 1) * kNB - 1 + g.kv) / kNB);
 }
-__device__ __forceinline__ bool handed_off(const Geo &g, int b) { return b >= 2 && p_first(g, b) <= b - 2; }
+// Block b passes through an update CTA (which applies panels p_first(b)..b-3).
+__device__ __forceinline__ bool handed_off(const Geo &g, int b) { return b >= 3 && p_first(g, b) <= b - 3; }
 
-// Block b (columns b*kNB ..) from AB into shared memory (kNB x ldab, AB layout).
+// Synchronisation and broadcast state.  Slots indexed [2] alternate with the
+// barrier count: a slot is rewritten only two barriers after it was published,
+// when every reader has passed the barrier in between.
+template <int RPT>
+struct WideShared {
+  unsigned long long key[2][RPT * kCW];
+  double piv[2][RPT * kCW][kNB];  // each warp's best candidate row, panel columns
+  int idx[2][RPT * kCW];
+  double row0[2][kNB];            // row j before the interchange, panel columns
+  double bu[2][kNB];              // lookahead: pivot row in the block's columns
+  double br0[2][kNB];             // lookahead: row j in the block's columns
+  unsigned bum[2];                // nonzero mask of bu
+  unsigned pivm[2][RPT * kCW];    // nonzero masks of piv
+  int pk[2][kNB];                 // pivot offsets of a panel, by panel parity
+  int zp[2][kNB];                 // exact zero pivot
+  unsigned long long mb_done[2];  // compute -> I/O: panel p finished (mb_done[p & 1])
+  unsigned long long mb_load[2];  // I/O -> compute: block b in shared memory (mb_load[b & 1])
+  int ok;
+  int info;
+};
+
+// ---- bounded waits ------------------------------------------------------------
+
+// Polls `ready` until it returns true; gives up (false) when *err is raised or
+// the cycle budget runs out (then raises *err itself).
+template <class F>
+__device__ __forceinline__ bool bounded_poll(F ready, int *err) {
+  if (ready()) return true;
+  const long long t0 = clock64();
+  for (unsigned it = 1;; ++it) {
+    if (ready()) return true;
+    if ((it & 15u) == 0u) {
+      if (ld_relaxed(err) != 0) return false;
+      if (clock64() - t0 > kSpinLimit) {
+        atomicExch(err, 1);
+        return false;
+      }
+    }
+  }
+}
+
+// All compute threads: thread 0 waits, the outcome is shared.
+template <int RPT, class F>
+__device__ bool compute_wait(F ready, int *err, WideShared<RPT> &sh) {
+  if (threadIdx.x == 0) sh.ok = bounded_poll(ready, err) ? 1 : 0;
+  bar_compute();
+  const bool ok = sh.ok != 0;
+  bar_compute();
+  return ok;
+}
+
+// I/O warp: lane 0 waits, the outcome is warp-uniform.
+template <class F>
+__device__ bool io_wait(F ready, int *err) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = bounded_poll(ready, err) ? 1 : 0;
+  ok = __shfl_sync(FULL, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+
+// ---- block transfers ------------------------------------------------------------
+// A block is kNB columns of AB (kNB * ldab doubles, the last block fewer).
 // first: the block's first read, so its fill rows 0..kl-1 are cleared (the
 // elimination clears every fill row before it starts).
-__device__ void load_block(const Geo &g, const double *AB, double *blk, int b, bool first) {
+
+__device__ void load_block(const Geo &g, const double *AB, double *blk, int b, bool first, int t, int nt) {
   const int c0 = b * kNB, nc = min(kNB, g.n - c0);
-  const long long tot = (long long)nc * g.ldab;
+  const int tot = nc * (int)g.ldab;
   const double *src = AB + (long long)c0 * g.ldab;
-  for (long long e = threadIdx.x; e < tot; e += kThreads) {
-    const long long r = e % g.ldab;
-    blk[e] = (first && r < g.kl) ? 0.0 : __ldcg(src + e);
+  if (first || !g.vec) {
+    for (int e = t; e < tot; e += nt) {
+      const int r = e % (int)g.ldab;
+      blk[e] = (first && r < g.kl) ? 0.0 : __ldcg(src + e);
+    }
+  } else {
+    for (int e = 2 * t; e + 1 < tot; e += 2 * nt)
+      reinterpret_cast<double2 *>(blk)[e >> 1] = __ldcg(reinterpret_cast<const double2 *>(src) + (e >> 1));
+    if ((tot & 1) && t == 0) blk[tot - 1] = __ldcg(src + tot - 1);
   }
-  __syncthreads();
 }
 
-__device__ void store_block(const Geo &g, double *AB, const double *blk, int b) {
+__device__ void store_block(const Geo &g, double *AB, const double *blk, int b, int t, int nt) {
   const int c0 = b * kNB, nc = min(kNB, g.n - c0);
-  const long long tot = (long long)nc * g.ldab;
+  const int tot = nc * (int)g.ldab;
   double *dst = AB + (long long)c0 * g.ldab;
-  for (long long e = threadIdx.x; e < tot; e += kThreads) dst[e] = blk[e];
-  __syncthreads();
+  if (!g.vec) {
+    for (int e = t; e < tot; e += nt) dst[e] = blk[e];
+  } else {
+    for (int e = 2 * t; e + 1 < tot; e += 2 * nt)
+      reinterpret_cast<double2 *>(dst)[e >> 1] = reinterpret_cast<const double2 *>(blk)[e >> 1];
+    if ((tot & 1) && t == 0) dst[tot - 1] = blk[tot - 1];
+  }
 }
 
-// Steps of panel p applied to block b (b > p): interchange, then the rank-1
-// update, column by column of the block, one step after the other.
-// s_l[k*kl + t-1] = multiplier l_{j+t, j} of column j = p*kNB + k; s_pk[k] = pivot
-// offset; s_zp[k] != 0 for an exactly zero pivot (no interchange, no update).
-__device__ void apply_panel(const Geo &g, double *blk, int b, int p, const double *s_l, const int *s_pk,
-                            const int *s_zp) {
+// I/O warp: copy of a handed-off block in 16-byte cp.async chunks (AB aligned).
+__device__ void io_prefetch_block(const Geo &g, const double *AB, double *blk, int b) {
+  const int lane = threadIdx.x & 31;
   const int c0 = b * kNB, nc = min(kNB, g.n - c0);
-  const long long ldab = g.ldab;
+  const int tot = nc * (int)g.ldab;
+  const double *src = AB + (long long)c0 * g.ldab;
+  for (int e = 2 * lane; e + 1 < tot; e += 64) {
+    const unsigned d = smem_addr(blk + e);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src + e) : "memory");
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+  if ((tot & 1) && lane == 0) blk[tot - 1] = __ldcg(src + tot - 1);
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
+// ---- one panel applied to a later block -----------------------------------------
+// Compute threads; thread i <-> row q*kNB + i (the rows of panel q's steps).
+// lr[r][k]: multiplier of the thread's row r at step k (0 if none).  The slot
+// parity `bpar` advances at each barrier.
+template <int RPT>
+__device__ void apply_panel(const Geo &g, double *blk, int b, int q, const double (&lr)[RPT][kNB], const int *pk,
+                            const int *zp, WideShared<RPT> &sh, int &bpar) {
+  const int tid = threadIdx.x;
+  const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
+  const int c0b = b * kNB, ncb = min(kNB, g.n - c0b);
+  const int ldab = (int)g.ldab;
+  double w[RPT][kNB];
+#pragma unroll
+  for (int r = 0; r < RPT; ++r) {
+    const int i = tid + r * kCT, row = c0q + i;
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) {
+      const int pos = g.kv + row - (c0b + d);
+      const bool ok = i < g.kl + kNB && row < g.n && d < ncb && pos >= 0;
+      w[r][d] = ok ? blk[d * ldab + pos] : 0.0;
+    }
+  }
+#pragma unroll
   for (int k = 0; k < kNB; ++k) {
-    const int j = p * kNB + k;
-    if (j >= g.n) break;
-    if (s_zp[k]) continue;  // uniform
-    const int km = min(g.kl, g.n - 1 - j);
-    const int pk = s_pk[k];
-    if (pk != 0) {
-      if (threadIdx.x < nc) {
-        const int c = c0 + threadIdx.x;
-        if (c <= j + g.kv) {  // beyond the reach of row j both entries are structural zeros
-          double *x = blk + threadIdx.x * ldab + (g.kv + j - c);
-          double *y = x + pk;
-          const double t0 = *x;
-          *x = *y;
-          *y = t0;
+    if (k >= ncq) break;
+    if (zp[k]) continue;  // uniform
+    const int j = c0q + k, km = min(g.kl, g.n - 1 - j), p = pk[k];
+    const int s = bpar;
+    bpar ^= 1;
+#pragma unroll
+    for (int r = 0; r < RPT; ++r) {
+      const int i = tid + r * kCT;
+      if (i == k + p) {
+#pragma unroll
+        for (int d = 0; d < kNB; ++d) sh.bu[s][d] = w[r][d];
+        sh.bum[s] = nz_mask(w[r]);
+      }
+      if (i == k) {
+#pragma unroll
+        for (int d = 0; d < kNB; ++d) sh.br0[s][d] = w[r][d];
+      }
+    }
+    bar_compute();
+    double u[kNB];
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) u[d] = sh.bu[s][d];
+    const unsigned um = sh.bum[s];
+#pragma unroll
+    for (int r = 0; r < RPT; ++r) {
+      const int i = tid + r * kCT;
+      if (i == k) {
+#pragma unroll
+        for (int d = 0; d < kNB; ++d) w[r][d] = u[d];
+      } else if (p != 0 && i == k + p) {
+#pragma unroll
+        for (int d = 0; d < kNB; ++d) w[r][d] = sh.br0[s][d];
+      }
+      if (i > k && i <= k + km) {
+        const double l = lr[r][k];
+#pragma unroll
+        for (int d = 0; d < kNB; ++d) w[r][d] = upd(l, u[d], w[r][d], (um >> d) & 1u);
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < RPT; ++r) {
+    const int i = tid + r * kCT, row = c0q + i;
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) {
+      const int pos = g.kv + row - (c0b + d);
+      if (i < g.kl + kNB && row < g.n && d < ncb && pos >= 0) blk[d * ldab + pos] = w[r][d];
+    }
+  }
+}
+
+// ---- panel factorisation (panel CTA compute threads) -----------------------------
+// Factors block p in place; records the pivot offsets and zero flags in
+// sh.pk/sh.zp[p & 1] and the multipliers in s_l (s_l[k*kl + t-1] = l_{j+t, j},
+// j = p*kNB + k).
+template <int RPT>
+__device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, WideShared<RPT> &sh, int &bpar,
+                             int &info) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int c0 = p * kNB, nc = min(kNB, g.n - c0);
+  const int ldab = (int)g.ldab;
+  const int pp = p & 1;
+  double v[RPT][kNB];
+#pragma unroll
+  for (int r = 0; r < RPT; ++r) {
+    const int i = tid + r * kCT, row = c0 + i;
+#pragma unroll
+    for (int k = 0; k < kNB; ++k) {
+      const bool ok = i < g.kl + kNB && row < g.n && k < nc && i - k <= g.kl;
+      v[r][k] = ok ? blk[k * ldab + g.kv + i - k] : 0.0;
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kNB; ++k) {
+    if (k >= nc) break;
+    const int j = c0 + k, km = min(g.kl, g.n - 1 - j);
+    const int s = bpar;
+    bpar ^= 1;
+#pragma unroll
+    for (int r = 0; r < RPT; ++r) {
+      const int i = tid + r * kCT, t = i - k;
+      const unsigned long long key = (t >= 0 && t <= km) ? pivot_key(v[r][k], t == 0) : 0ull;
+      unsigned long long kmax;
+      const int wl = warp_first_max(key, &kmax);
+      if (lane == wl) {
+        sh.key[s][r * kCW + warp] = kmax;
+        sh.idx[s][r * kCW + warp] = i;
+#pragma unroll
+        for (int d = 0; d < kNB; ++d) sh.piv[s][r * kCW + warp][d] = v[r][d];
+        sh.pivm[s][r * kCW + warp] = nz_mask(v[r]);
+      }
+      if (i == k) {
+#pragma unroll
+        for (int d = 0; d < kNB; ++d) sh.row0[s][d] = v[r][d];
+      }
+    }
+    bar_compute();
+    // the first largest key over the partials, which are in row order
+    unsigned long long best = sh.key[s][0];
+    int wb = 0;
+#pragma unroll
+    for (int x = 1; x < RPT * kCW; ++x) {
+      const unsigned long long kx = sh.key[s][x];
+      if (kx > best) {
+        best = kx;
+        wb = x;
+      }
+    }
+    const int p_off = sh.idx[s][wb] - k;
+    double u[kNB];
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) u[d] = sh.piv[s][wb][d];
+    const unsigned um = sh.pivm[s][wb];
+    const bool zero = ((um >> k) & 1u) == 0u;
+    if (tid == 0) {
+      sh.pk[pp][k] = p_off;
+      sh.zp[pp][k] = zero ? 1 : 0;
+      if (zero && info == 0) info = j + 1;
+    }
+    if (!zero) {
+      const double rc = rcp_rn(u[k]);
+#pragma unroll
+      for (int r = 0; r < RPT; ++r) {
+        const int i = tid + r * kCT;
+        if (i == k) {
+#pragma unroll
+          for (int d = 0; d < kNB; ++d)
+            if (d >= k) v[r][d] = u[d];
+        } else if (p_off != 0 && i == k + p_off) {
+#pragma unroll
+          for (int d = 0; d < kNB; ++d)
+            if (d >= k) v[r][d] = sh.row0[s][d];
+        }
+        if (i > k && i <= k + km) {
+          const double l = v[r][k] * rc;
+          v[r][k] = l;
+#pragma unroll
+          for (int d = 0; d < kNB; ++d)
+            if (d > k) v[r][d] = upd(l, u[d], v[r][d], (um >> d) & 1u);
         }
       }
-      __syncthreads();
     }
-    if (km > 0) {
-      const int tot = km * nc;
-      for (int e = threadIdx.x; e < tot; e += kThreads) {
-        const int cc = e / km, t = 1 + (e - cc * km);
-        const int c = c0 + cc;
-        if (c > j + g.kv) continue;
-        double *col = blk + cc * ldab + (g.kv + j - c);
-        const double u = col[0];
-        if (nz(u)) col[t] = fma(-s_l[k * g.kl + t - 1], u, col[t]);
-      }
-      __syncthreads();
+  }
+#pragma unroll
+  for (int r = 0; r < RPT; ++r) {
+    const int i = tid + r * kCT, row = c0 + i;
+#pragma unroll
+    for (int k = 0; k < kNB; ++k) {
+      if (i < g.kl + kNB && row < g.n && k < nc && i - k <= g.kl) blk[k * ldab + g.kv + i - k] = v[r][k];
+      const int t = i - k;
+      if (k < nc && t >= 1 && t <= min(g.kl, g.n - 1 - (c0 + k))) s_l[k * g.kl + t - 1] = v[r][k];
     }
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(int n, int kl, int ku, double *__restrict__ AB,
-                                                              long long ldab, int *__restrict__ ipiv,
+template <int RPT>
+__global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__restrict__ AB, int *__restrict__ ipiv,
                                                               int *__restrict__ d_info, int *__restrict__ flags) {
-  extern __shared__ double smem[];
-  __shared__ KeyIdx s_red[kThreads / 32];
-  __shared__ int s_pk[kNB], s_zp[kNB], s_ok, s_p;
-  Geo g;
-  g.n = n;
-  g.kl = kl;
-  g.ku = ku;
-  g.kv = kl + ku;
-  g.ldab = ldab;
-  g.npan = (n + kNB - 1) / kNB;
+  extern __shared__ __align__(16) double smem[];
+  __shared__ WideShared<RPT> sh;
   int *err = flags;
   int *panel_ready = flags + 2;
   int *block_ready = flags + 2 + g.npan;
-  double *s_l = smem;                        // kNB * kl multipliers of the current panel
-  double *blocks = smem + (size_t)kNB * kl;  // kMaxActive blocks of kNB * ldab
-  const long long bsz = (long long)kNB * ldab;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long bsz = (long long)kNB * g.ldab;
+  double *blocks = smem;                              // kPanelBufs (panel CTA) / kMaxActive blocks
+  double *s_lbase = smem + (size_t)kPanelBufs * bsz;  // 2 panels of kNB * kl multipliers
+  const int tid = threadIdx.x, warp = tid >> 5;
+
+  if (blockIdx.x == 0 && tid == 0) {
+    mbar_init(&sh.mb_done[0], 1);
+    mbar_init(&sh.mb_done[1], 1);
+    mbar_init(&sh.mb_load[0], 1);
+    mbar_init(&sh.mb_load[1], 1);
+    sh.info = 0;
+  }
+  __syncthreads();
 
   if (blockIdx.x == 0) {
-    // ---------------- panel CTA ----------------
-    int info = 0;
-    double *cur = blocks, *nxt = blocks + bsz;
-    load_block(g, AB, cur, 0, true);
-    for (int p = 0; p < g.npan; ++p) {
-      const int c0 = p * kNB, nc = min(kNB, n - c0);
-      for (int k = 0; k < nc; ++k) {
-        const int j = c0 + k;
-        const int km = min(kl, n - 1 - j);
-        double *col = cur + k * ldab + g.kv;  // col[t] = entry (j+t, j)
-        KeyIdx best{0ull, LLONG_MAX};
-        for (int t = threadIdx.x; t <= km; t += kThreads) best = better(best, KeyIdx{abs_key(col[t]), t});
-        best = warp_reduce_keyidx(best);
-        if (lane == 0) s_red[warp] = best;
-        __syncthreads();
-        if (warp == 0) {
-          KeyIdx v = lane < kThreads / 32 ? s_red[lane] : KeyIdx{0ull, LLONG_MAX};
-          v = warp_reduce_keyidx(v);
-          if (lane == 0) s_p = (int)v.idx;
-        }
-        __syncthreads();
-        const int pr = s_p;
-        const double pv = col[pr];
-        const bool zp = !nz(pv);
-        if (threadIdx.x == 0) {
-          ipiv[j] = j + pr + 1;
-          s_pk[k] = pr;
-          s_zp[k] = zp ? 1 : 0;
-        }
-        if (zp) {
-          if (info == 0) info = j + 1;
-          __syncthreads();
-          continue;
-        }
-        if (pr != 0) {
-          if (threadIdx.x < nc - k && threadIdx.x <= g.kv) {  // columns j .. block end, rows j and j+pr
-            const int c = j + threadIdx.x;
-            double *x = cur + (c - c0) * ldab + (g.kv + j - c);
-            const double t0 = x[0];
-            x[0] = x[pr];
-            x[pr] = t0;
+    if (warp < kCW) {
+      // ---------------- panel CTA: compute warps ----------------
+      int info = 0, bpar = 0;
+      load_block(g, AB, blocks, 0, true, tid, kCT);
+      if (g.npan > 1) load_block(g, AB, blocks + bsz, 1, true, tid, kCT);
+      bar_compute();
+      for (int p = 0; p < g.npan; ++p) {
+        double *cur = blocks + (long long)(p % kPanelBufs) * bsz;
+        double *s_l = s_lbase + (size_t)(p & 1) * kNB * g.kl;
+        factor_panel<RPT>(g, cur, p, s_l, sh, bpar, info);
+        if (tid == 0) sh.info = info;
+        bar_compute();
+        if (tid == 0) mbar_arrive(&sh.mb_done[p & 1]);
+        if (p + 1 < g.npan) {
+          const int b = p + 1;
+          double *nxt = blocks + (long long)(b % kPanelBufs) * bsz;
+          if (b >= 2) {
+            unsigned long long *mb = &sh.mb_load[b & 1];
+            const unsigned par = (unsigned)((b - 2) >> 1) & 1u;
+            if (!compute_wait<RPT>([&] { return mbar_try_wait(mb, par); }, err, sh)) break;
           }
-          __syncthreads();
-        }
-        const double r = rcp_rn(pv);
-        for (int t = 1 + threadIdx.x; t <= km; t += kThreads) col[t] *= r;
-        __syncthreads();
-        const int rest = min(nc - 1 - k, g.kv);
-        if (rest > 0 && km > 0) {
-          for (int e = threadIdx.x; e < km * rest; e += kThreads) {
-            const int cc = e / km, t = 1 + (e - cc * km);
-            const int c = j + 1 + cc;
-            double *cj = cur + (c - c0) * ldab + (g.kv + j - c);
-            const double u = cj[0];
-            if (nz(u)) cj[t] = fma(-col[t], u, cj[t]);
+          double lr[RPT][kNB];
+          for (int q = p - 1; q <= p; ++q) {
+            if (q < 0 || q < p_first(g, b)) continue;  // uniform
+            const double *ql = s_lbase + (size_t)(q & 1) * kNB * g.kl;
+            const int c0q = q * kNB;
+#pragma unroll
+            for (int r = 0; r < RPT; ++r) {
+              const int i = tid + r * kCT;
+#pragma unroll
+              for (int k = 0; k < kNB; ++k) {
+                const int t = i - k;
+                lr[r][k] = (c0q + k < g.n && t >= 1 && t <= min(g.kl, g.n - 1 - (c0q + k))) ? ql[k * g.kl + t - 1]
+                                                                                             : 0.0;
+              }
+            }
+            apply_panel<RPT>(g, nxt, b, q, lr, sh.pk[q & 1], sh.zp[q & 1], sh, bpar);
+            bar_compute();
           }
-          __syncthreads();
         }
       }
-      // publish panel p: the block to AB (U rows, multipliers, pivots already out)
-      for (int e = threadIdx.x; e < kNB * kl; e += kThreads) {
-        const int k = e / kl, t = 1 + (e - k * kl);
-        s_l[e] = (k < nc && t <= min(kl, n - 1 - (c0 + k))) ? cur[k * ldab + g.kv + t] : 0.0;
+    } else {
+      // ---------------- panel CTA: I/O warp ----------------
+      const int lane = tid & 31;
+      for (int p = 0; p < g.npan; ++p) {
+        unsigned long long *mb = &sh.mb_done[p & 1];
+        const unsigned par = (unsigned)(p >> 1) & 1u;
+        if (!io_wait([&] { return mbar_try_wait(mb, par); }, err)) break;
+        const int c0 = p * kNB, nc = min(kNB, g.n - c0);
+        store_block(g, AB, blocks + (long long)(p % kPanelBufs) * bsz, p, lane, 32);
+        if (lane < nc) ipiv[c0 + lane] = c0 + lane + sh.pk[p & 1][lane] + 1;
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) st_release(panel_ready + p, 1);
+        const int b = p + 2;
+        if (b < g.npan) {
+          double *dst = blocks + (long long)(b % kPanelBufs) * bsz;
+          if (handed_off(g, b)) {
+            const int *f = block_ready + b;
+            if (!io_wait([&] { return ld_acquire(f) != 0; }, err)) break;
+            if (g.vec) {
+              io_prefetch_block(g, AB, dst, b);
+            } else {
+              load_block(g, AB, dst, b, false, lane, 32);
+            }
+          } else {
+            load_block(g, AB, dst, b, true, lane, 32);
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sh.mb_load[b & 1]);
+        }
       }
-      store_block(g, AB, cur, p);
-      cta_signal(panel_ready + p);
-      if (p + 1 < g.npan) {
-        const bool ho = handed_off(g, p + 1);
-        if (ho && !cta_wait(block_ready + p + 1, err, &s_ok)) break;
-        load_block(g, AB, nxt, p + 1, !ho);
-        apply_panel(g, nxt, p + 1, p, s_l, s_pk, s_zp);
-        double *tmp = cur;
-        cur = nxt;
-        nxt = tmp;
-      }
-      __syncthreads();
+      // info is final once the last panel is done; the status reflects every CTA's waits
+      if (lane == 0) *d_info = ld_acquire(err) ? -BANDLU_ERR_TIMEOUT : sh.info;
     }
-    if (threadIdx.x == 0) *d_info = ld_acquire(err) ? -BANDLU_ERR_TIMEOUT : info;
   } else {
     // ---------------- update CTAs ----------------
+    if (warp >= kCW) return;
     const int G = gridDim.x - 1, u = blockIdx.x - 1;
-    for (int p = 0; p + 2 < g.npan; ++p) {
-      // owned blocks that panel p updates here: b in [p+2, b_last(p)], b = 2 + u (mod G)
-      const int lo = p + 2, hi = b_last(g, p);
-      int b0 = lo + ((u - (lo - 2)) % G + G) % G;
+    int bpar = 0;
+    for (int p = 0; p + 3 < g.npan; ++p) {
+      // owned blocks that panel p updates here: b in [p+3, b_last(p)], b = 3 + u (mod G)
+      const int lo = p + 3, hi = b_last(g, p);
+      const int b0 = lo + ((u - (lo - 3)) % G + G) % G;
       if (b0 > hi) continue;
-      if (!cta_wait(panel_ready + p, err, &s_ok)) break;
-      // panel p's multipliers and pivots (written by the panel CTA before panel_ready[p])
-      const int c0 = p * kNB, nc = min(kNB, n - c0);
-      for (int e = threadIdx.x; e < kNB * kl; e += kThreads) {
-        const int k = e / kl, t = 1 + (e - k * kl);
-        s_l[e] = (k < nc && t <= min(kl, n - 1 - (c0 + k)))
-                     ? __ldcg(AB + (long long)(c0 + k) * ldab + g.kv + t)
-                     : 0.0;
+      const int *f = panel_ready + p;
+      if (!compute_wait<RPT>([&] { return ld_acquire(f) != 0; }, err, sh)) break;
+      const int c0q = p * kNB, ncq = min(kNB, g.n - c0q);
+      if (tid < kNB) {
+        const int k = tid;
+        sh.pk[0][k] = k < ncq ? __ldcg(ipiv + c0q + k) - 1 - (c0q + k) : 0;
+        sh.zp[0][k] = k < ncq ? (nz(__ldcg(AB + (long long)(c0q + k) * g.ldab + g.kv)) ? 0 : 1) : 1;
       }
-      if (threadIdx.x < kNB) {
-        const int k = threadIdx.x;
-        s_pk[k] = k < nc ? __ldcg(ipiv + c0 + k) - 1 - (c0 + k) : 0;
-        s_zp[k] = k < nc ? (nz(__ldcg(AB + (long long)(c0 + k) * ldab + g.kv)) ? 0 : 1) : 1;
-      }
-      __syncthreads();
-      for (int b = b0; b <= hi; b += G) {
-        double *blk = blocks + (long long)((b - 2) / G % kMaxActive) * bsz;
-        const int pf = p_first(g, b);
-        if (p == pf) load_block(g, AB, blk, b, true);
-        apply_panel(g, blk, b, p, s_l, s_pk, s_zp);
-        if (p == b - 2) {
-          store_block(g, AB, blk, b);
-          cta_signal(block_ready + b);
+      double lr[RPT][kNB];
+#pragma unroll
+      for (int r = 0; r < RPT; ++r) {
+        const int i = tid + r * kCT;
+#pragma unroll
+        for (int k = 0; k < kNB; ++k) {
+          const int t = i - k;
+          lr[r][k] = (k < ncq && t >= 1 && t <= min(g.kl, g.n - 1 - (c0q + k)))
+                         ? __ldcg(AB + (long long)(c0q + k) * g.ldab + g.kv + t)
+                         : 0.0;
         }
       }
-      __syncthreads();
+      bar_compute();
+      for (int b = b0; b <= hi; b += G) {
+        double *blk = blocks + (long long)(((b - 3) / G) % kMaxActive) * bsz;
+        if (p == p_first(g, b)) {
+          load_block(g, AB, blk, b, true, tid, kCT);
+          bar_compute();
+        }
+        apply_panel<RPT>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh, bpar);
+        bar_compute();
+        if (p == b - 3) {
+          store_block(g, AB, blk, b, tid, kCT);
+          __threadfence();
+          bar_compute();
+          if (tid == 0) st_release(block_ready + b, 1);
+        }
+      }
     }
   }
 }
 
-}  // namespace
-
-// Launch conditions: every update CTA holds at most kMaxActive blocks at once
-// and both roles fit in shared memory.  Returns BANDLU_ERR_UNSUPPORTED_SHAPE
-// (a positive code never seen by callers) when the shape does not qualify.
-int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s,
-                      bool *used) {
-  *used = false;
-  if (n < 3 * kNB || kl < 1) return BANDLU_OK;
-  int dev = 0, sms = 0, coop = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return BANDLU_ERR_CUDA;
-  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
-  if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
-  if (!coop || sms < 2) return BANDLU_OK;
-  const long long kv = (long long)kl + ku;
-  const size_t smem = ((size_t)kNB * kl + (size_t)kMaxActive * kNB * (size_t)ldab) * sizeof(double);
-  if (smem > 200 * 1024) return BANDLU_OK;
-  const int G = sms - 1;
-  const long long span = (kv - 1) / kNB + 2;  // blocks one panel updates, at most
-  if (span > (long long)kMaxActive * G) return BANDLU_OK;
+// Returns BANDLU_OK after a launch, BANDLU_NOT_BANDED when the kernel cannot be
+// made resident (the caller then takes another kernel), or BANDLU_ERR_CUDA.
+template <int RPT>
+int launch_rpt(const Geo &g, int grid, size_t smem, double *AB, int *ipiv, int *d_info, int *flags, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    if (cudaFuncSetAttribute(k_gbtrf_wide, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
+    if (cudaFuncSetAttribute(k_gbtrf_wide<RPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
         cudaSuccess)
       return BANDLU_ERR_CUDA;
     attr = true;
   }
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_gbtrf_wide, kThreads, smem) != cudaSuccess)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_gbtrf_wide<RPT>, kThreads, smem) != cudaSuccess)
     return BANDLU_ERR_CUDA;
-  if (per_sm < 1) return BANDLU_OK;
+  if (per_sm < 1) return BANDLU_NOT_BANDED;
+  Geo gg = g;
+  void *args[] = {&gg, &AB, &ipiv, &d_info, &flags};
+  if (cudaLaunchCooperativeKernel((const void *)k_gbtrf_wide<RPT>, dim3(grid), dim3(kThreads), args, smem, s) !=
+      cudaSuccess)
+    return BANDLU_ERR_CUDA;
+  return BANDLU_OK;
+}
+
+}  // namespace
+
+// Launch conditions: kv >= 2*kNB, at most 4 panel rows per compute thread,
+// shared memory for three blocks and two panels of multipliers, and an update
+// CTA never holding more than kMaxActive blocks.  *used = false when the shape
+// does not qualify (the caller then takes another kernel).
+int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s,
+                      bool *used) {
+  *used = false;
+  const long long kv = (long long)kl + ku;
+  if (n < 4 * kNB || n > INT_MAX / 2 || kl < 1 || kv < 2 * kNB || ldab > INT_MAX / kNB) return BANDLU_OK;
+  const int rpt = (kl + kNB + kCT - 1) / kCT;
+  if (rpt > 4) return BANDLU_OK;
+  const size_t smem = ((size_t)kPanelBufs * kNB * (size_t)ldab + 2 * (size_t)kNB * kl) * sizeof(double);
+  if (smem > 200 * 1024) return BANDLU_OK;
+  int dev = 0, sms = 0, coop = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (!coop || sms < 2) return BANDLU_OK;
+  const int G = sms - 1;
+  const long long span = (kv + 3) / kNB + 1;  // blocks one panel updates, at most
+  if (span > (long long)kMaxActive * G) return BANDLU_OK;
+  Geo g;
+  g.n = (int)n;
+  g.kl = kl;
+  g.ku = ku;
+  g.kv = (int)kv;
+  g.ldab = ldab;
+  g.npan = (int)((n + kNB - 1) / kNB);
+  g.vec = (reinterpret_cast<uintptr_t>(AB) & 15u) == 0;
   // scratch: error flag, spare, panel_ready[npan], block_ready[npan]
-  const long long npan = (n + kNB - 1) / kNB;
-  const size_t fbytes = (size_t)(2 + 2 * npan) * sizeof(int);
+  const size_t fbytes = (size_t)(2 + 2 * (size_t)g.npan) * sizeof(int);
   int *flags = nullptr;
   if (cudaMallocAsync(reinterpret_cast<void **>(&flags), fbytes, s) != cudaSuccess) return BANDLU_ERR_CUDA;
-  if (cudaMemsetAsync(flags, 0, fbytes, s) != cudaSuccess) return BANDLU_ERR_CUDA;
-  int nn = (int)n, kkl = kl, kku = ku;
-  long long lld = ldab;
-  void *args[] = {&nn, &kkl, &kku, &AB, &lld, &ipiv, &d_info, &flags};
-  const cudaError_t e = cudaLaunchCooperativeKernel((const void *)k_gbtrf_wide, dim3(sms), dim3(kThreads), args,
-                                                    smem, s);
-  cudaFreeAsync(flags, s);
-  if (e != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (cudaMemsetAsync(flags, 0, fbytes, s) != cudaSuccess) {
+    cudaFreeAsync(flags, s);
+    return BANDLU_ERR_CUDA;
+  }
+  int rc;
+  if (rpt == 1)
+    rc = launch_rpt<1>(g, sms, smem, AB, ipiv, d_info, flags, s);
+  else if (rpt == 2)
+    rc = launch_rpt<2>(g, sms, smem, AB, ipiv, d_info, flags, s);
+  else
+    rc = launch_rpt<4>(g, sms, smem, AB, ipiv, d_info, flags, s);
+  if (cudaFreeAsync(flags, s) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (rc == BANDLU_NOT_BANDED) return BANDLU_OK;
+  if (rc != BANDLU_OK) return rc;
   *used = true;
   return BANDLU_OK;
 }

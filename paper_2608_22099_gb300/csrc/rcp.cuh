@@ -103,11 +103,22 @@ __host__ __device__ __forceinline__ double rcp_rn_fast(double b, bool *special) 
   return bitsd(frac == 0 ? pbits : rbits);
 }
 
+#ifdef __CUDACC__
+// Out of line, so that the rarely taken division is never if-converted (an
+// unconditional FP64 division in every thread costs more than the reciprocal).
+__device__ __noinline__ static double rcp_division(double b) { return 1.0 / b; }
+#endif
+
 // Correctly rounded 1/b (IEEE binary64, round to nearest even).
 __host__ __device__ __forceinline__ double rcp_rn(double b) {
   bool special;
-  const double r = rcp_rn_fast(b, &special);
-  return special ? 1.0 / b : r;
+  double r = rcp_rn_fast(b, &special);
+#ifdef __CUDA_ARCH__
+  if (special) r = rcp_division(b);
+#else
+  if (special) r = 1.0 / b;
+#endif
+  return r;
 }
 
 }  // namespace bandlu
