@@ -131,10 +131,10 @@ __device__ int warp_gbtrf(double *ab, int ldab, int n, int kl, int ku, int *ipiv
     if (km < 32) {
       const double x = lane <= km ? col[kv + lane] : 0.0;
       bool allz;
-      p = warp_argmax_first_z(lane <= km ? abs_key(x) : 0ull, &allz);
+      p = warp_argmax_first_z(lane <= km ? pivot_abs_key(x, lane == 0) : 0ull, &allz);
     } else {
       KeyIdx best{0ull, LLONG_MAX};
-      for (int t = lane; t <= km; t += 32) best = better(best, KeyIdx{abs_key(col[kv + t]), t});
+      for (int t = lane; t <= km; t += 32) best = better(best, KeyIdx{pivot_abs_key(col[kv + t], t == 0), t});
       p = (int)warp_reduce_keyidx(best).idx;
     }
     const double pv = col[kv + p];

@@ -21,9 +21,16 @@ __device__ __forceinline__ bool nz(double x) {
   return ((((unsigned)__double2hiint(x)) << 1) | (unsigned)__double2loint(x)) != 0u;
 }
 
-// |x| as an unsigned key: for non-NaN doubles, |x| < |y| iff key(x) < key(y).
-__device__ __forceinline__ unsigned long long abs_key(double x) {
-  return (unsigned long long)__double_as_longlong(x) & 0x7fffffffffffffffull;
+// Pivot-search key of a candidate: for non-NaN doubles |x| < |y| iff
+// key(x) < key(y).  The xGBTRF comparison order starts its running best at the
+// first candidate and replaces it only by a strictly larger modulus, which a
+// NaN never is: so a NaN gets the largest key as the first candidate (it is
+// kept) and the key of zero otherwise (with the first-index rule on ties it is
+// never chosen over an earlier candidate).
+__device__ __forceinline__ unsigned long long pivot_abs_key(double x, bool first) {
+  const unsigned hi = (unsigned)__double2hiint(x) & 0x7fffffffu, lo = (unsigned)__double2loint(x);
+  const bool nan = hi > 0x7ff00000u || (hi == 0x7ff00000u && lo != 0u);
+  return nan ? (first ? ~0ull : 0ull) : (((unsigned long long)hi << 32) | lo);
 }
 
 // First lane holding the largest key among all 32 lanes (ties -> lowest lane).

@@ -171,7 +171,7 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
       const int km = min(kl, n - 1 - j);
       const bool valid = lane <= km;
       bool zp;  // exact zero pivot (then p == 0)
-      const int p = warp_argmax_first_z(valid ? abs_key(cur) : 0ull, &zp);
+      const int p = warp_argmax_first_z(valid ? pivot_abs_key(cur, lane == 0) : 0ull, &zp);
       // interchange rows j and j+p: lanes 0 and p trade their values and slots
       const int src = lane == 0 ? p : (lane == p ? 0 : lane);
       slot_reg = __shfl_sync(FULL, slot_reg, src);
@@ -377,7 +377,7 @@ __global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int
     const long long km = min((long long)kl, n - 1 - j);
     double *colj = AB + j * ldab;
     KeyIdx best{0ull, LLONG_MAX};
-    for (long long t = tid; t <= km; t += B) best = better(best, KeyIdx{abs_key(colj[kv + t]), t});
+    for (long long t = tid; t <= km; t += B) best = better(best, KeyIdx{pivot_abs_key(colj[kv + t], t == 0), t});
     best = warp_reduce_keyidx(best);
     if (lane == 0) s_red[warp] = best;
     __syncthreads();

@@ -248,6 +248,49 @@ def test_gbtrf_wide_deterministic():
 
 
 # --------------------------------------------------------------------------------------------
+# NaN candidates: the pivot rule of the comparison order (a NaN is kept only as the first
+# candidate), in every kernel
+# --------------------------------------------------------------------------------------------
+
+def assert_parity_with_nan(AB, ipiv, info, ABr, ipr, infr):
+    assert info == infr and np.array_equal(ipiv, ipr)
+    nan_g, nan_r = np.isnan(AB), np.isnan(ABr)
+    assert np.array_equal(nan_g, nan_r)                  # NaN payloads may differ; positions may not
+    assert np.array_equal(AB[~nan_g].view(np.int64), ABr[~nan_r].view(np.int64))
+
+
+def plant_nans(A, kl, ku):
+    n = A.shape[0]
+    r0 = max(0, n - 60)
+    for (i, j) in ((r0 + 3, r0), (r0 + 1, r0 + 1), (r0 + 9, r0 + 7), (r0 + 12, r0 + 12)):
+        if i < n and j < n and -ku <= j - i <= kl and i - j <= kl:
+            A[i, j] = np.nan
+    return A
+
+
+@pytest.mark.parametrize("n,kl,ku", [(300, 5, 4), (200, 27, 3), (400, 40, 30), (14, 30, 2)])
+def test_gbtrf_nan_candidates(n, kl, ku):
+    A = plant_nans(banded(n, kl, ku, seed=n + kl, dist="normal").numpy(), kl, ku)
+    AB = oracle.dense_to_band(A, kl, ku)
+    ref = oracle.gbtrf(AB, kl, ku)
+    assert_parity_with_nan(*gbtrf_gpu(AB, kl, ku), ref[0], ref[1], ref[2])
+
+
+@pytest.mark.parametrize("n,kl,ku", [(64, 3, 3), (100, 40, 8)])
+def test_batched_nan_candidates(n, kl, ku):
+    batch = 6
+    A = torch.stack([torch.from_numpy(plant_nans(banded(n, kl, ku, seed=b).numpy(), kl, ku)) for b in range(batch)])
+    ldab = 2 * kl + ku + 1
+    got = run_batched(A, ldab)
+    ref = oracle.dispatch_lu_batched(A.numpy(), ldab)
+    for key in ("kl", "ku", "status", "info"):
+        assert np.array_equal(got[key], ref[key]), key
+    for b in range(batch):
+        assert_parity_with_nan(got["AB"][b], got["ipiv"][b], int(got["info"][b]), ref["AB"][b], ref["ipiv"][b],
+                               int(ref["info"][b]))
+
+
+# --------------------------------------------------------------------------------------------
 # dispatch_lu and dispatch_lu_batched
 # --------------------------------------------------------------------------------------------
 

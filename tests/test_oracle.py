@@ -326,6 +326,23 @@ def test_gbtrf_zero_pivot_sets_info_and_continues(oracle_mod):
     assert info2 == 3                                      # the first zero pivot is reported
 
 
+def test_gbtrf_pivot_comparison_order_with_nan(oracle_mod):
+    # The pivot is the first candidate of largest modulus in the comparison order
+    # of the running maximum (LAPACK's IDAMAX rule): a later candidate replaces the
+    # running best only if strictly larger, which a NaN never is.
+    n, kl, ku = 3, 2, 1
+    def piv(col0):
+        A = np.eye(n) * 3.0
+        A[:, 0] = col0
+        A[0, 1] = 0.5
+        ABf, ipiv, info, _ = oracle_mod.gbtrf(oracle_mod.dense_to_band(A, kl, ku), kl, ku)
+        return int(ipiv[0]), info
+    assert piv([1.0, np.nan, 2.0]) == (3, 0)          # NaN skipped, 2 > 1 taken
+    assert piv([np.nan, 5.0, -7.0]) == (1, 0)         # a NaN first candidate is kept
+    assert piv([0.0, np.nan, 0.0]) == (1, 1)          # NaN never beats zero: zero pivot
+    assert piv([-0.0, 0.0, np.inf])[0] == 3           # signed zeros tie, infinity wins
+
+
 def test_gbtrf_invariants_and_backward_error(oracle_mod):
     rng = np.random.default_rng(12)
     for trial in range(40):
