@@ -170,6 +170,10 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
     for (int j = 0; j < n; ++j) {
       const int km = min(kl, n - 1 - j);
       const bool valid = lane <= km;
+      // every lane forms the reciprocal of its own candidate while the argmax
+      // runs; the pivot's is then taken from the winning lane
+      bool myspec;
+      const double myr = rcp_rn_fast(cur, &myspec);  // integer pipes
       bool zp;  // exact zero pivot (then p == 0)
       const int p = warp_argmax_first_z(valid ? pivot_abs_key(cur, lane == 0) : 0ull, &zp);
       // interchange rows j and j+p: lanes 0 and p trade their values and slots
@@ -180,10 +184,9 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
       if (j >= 1 && !BAR_SYNC(kBarCol, 64, ph_col)) break;
       double v = 0.0;
       if (j + 1 < n && lane <= kl + 1 && j + lane < n) v = W[slot_reg * CS + qn];
-      const double pv = __shfl_sync(FULL, cur, p);
-      bool rspec;
-      double r = rcp_rn_fast(zp ? 1.5 : pv, &rspec);  // integer pipes
-      if (rspec && !zp) r = div_slow(pv);               // subnormal / huge pivot: plain division
+      double r = __shfl_sync(FULL, myr, p);
+      const bool rspec = __shfl_sync(FULL, myspec ? 1 : 0, p) != 0;
+      if (rspec && !zp) r = div_slow(__shfl_sync(FULL, cur, p));  // subnormal / huge pivot: plain division
       cur = __shfl_sync(FULL, cur, src);
       // U(j, j+1); when kv == 0 (diagonal matrix) column j+1 lies outside row j's band
       const double u = kv >= 1 ? __shfl_sync(FULL, v, 0) : 0.0;
