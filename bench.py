@@ -11,11 +11,14 @@ ranks time).  N > 1 runs independent replicas (the single-matrix path has no
 data-parallel split), one per GPU.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py --workload NAME [--steps K]     per-stage report of a named workload
+  python bench.py --custom N KL KU [BATCH]        the same report for a synthetic shape
 """
 from __future__ import annotations
 
 import argparse
 import atexit
+import hashlib
 import json
 import os
 import statistics
@@ -33,6 +36,45 @@ METRIC = "dispatch_lu time & GFLOP/s per matrix; detection HBM GB/s vs peak; spe
 WORKLOAD = "n4096_kl16_ku16"
 FP64_PEAK_GFLOPS = 1250.0  # nominal dense FP64 of one GB300 (152 SMs x 2 DFMA/clk x 2 flop x ~2.07 GHz)
 FALLBACK_HBM_GBS = 6800.0
+
+
+# Sources of each kernel: a DRAM-traffic figure taken by ncu is valid only while
+# their hash is the one recorded beside it under profiles/.
+KERNEL_SOURCES = {
+    "k_gbtrf_window": ["gbtrf.cu", "common.cuh", "rcp.cuh", "sync.cuh"],
+    "k_detect_vec": ["detect.cu", "common.cuh"],
+    "k_dense_to_band_tiled": ["convert.cu", "common.cuh"],
+}
+
+
+def kernel_source_hash(kernel: str) -> str:
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2608_22099_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str):
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the
+    committed ncu summary of the kernel, or None when there is none or the kernel's
+    sources changed since it was captured."""
+    pdir = os.path.join(ROOT, "profiles")
+    if not os.path.isdir(pdir):
+        return None
+    want = kernel_source_hash(kernel)
+    for fn in sorted(os.listdir(pdir)):
+        if not fn.startswith(kernel + "_") or not fn.endswith(".md"):
+            continue
+        fields = {}
+        with open(os.path.join(pdir, fn)) as f:
+            for line in f:
+                if line.startswith("traffic_bytes_per_launch:") or line.startswith("source_sha256:"):
+                    k, v = line.split(":", 1)
+                    fields[k.strip()] = v.strip()
+        if fields.get("source_sha256") == want and "traffic_bytes_per_launch" in fields:
+            return float(fields["traffic_bytes_per_launch"])
+    return None
 
 
 def load_peaks():
@@ -282,16 +324,19 @@ def run_ours(args):
     if dominant == "gbtrf":
         achieved = flops / t_gbtrf / 1e9
         roofline = {"bound": "alu", "achieved": achieved / 1e3, "peak": FP64_PEAK_GFLOPS / 1e3, "unit": "TFLOP/s",
-                    "frac": achieved / FP64_PEAK_GFLOPS, "traffic": None, "kernel": "k_gbtrf_window",
+                    "frac": achieved / FP64_PEAK_GFLOPS, "traffic": profiled_traffic("k_gbtrf_window"),
+                    "kernel": "k_gbtrf_window",
                     "peak_source": "nominal FP64 (152 SMs x 2 DFMA/clk x 2 flop x 2.07 GHz)",
                     "note": "one matrix is one serial pivot chain on one SM: latency-bound, see ns_per_column"}
     elif dominant == "detect":
         roofline = {"bound": "hbm", "achieved": detect_bytes / t_detect / 1e9, "peak": hbm_peak, "unit": "GB/s",
-                    "frac": detect_bytes / t_detect / 1e9 / hbm_peak, "traffic": None, "kernel": "k_detect_vec",
+                    "frac": detect_bytes / t_detect / 1e9 / hbm_peak, "traffic": profiled_traffic("k_detect_vec"),
+                    "kernel": "k_detect_vec",
                     "peak_source": hbm_src}
     else:
         roofline = {"bound": "hbm", "achieved": convert_bytes / t_convert / 1e9, "peak": hbm_peak, "unit": "GB/s",
-                    "frac": convert_bytes / t_convert / 1e9 / hbm_peak, "traffic": None,
+                    "frac": convert_bytes / t_convert / 1e9 / hbm_peak,
+                    "traffic": profiled_traffic("k_dense_to_band_tiled"),
                     "kernel": "k_dense_to_band_tiled", "peak_source": hbm_src}
 
     # end to end: pinned host input -> device, dispatch_lu, factors back to pinned host memory
@@ -367,9 +412,15 @@ def run_workload_report(args):
     import torch
 
     from paper_2608_22099_gb300 import bandlu
-    from paper_2608_22099_gb300.workloads import WORKLOADS, make_workload
+    from paper_2608_22099_gb300.workloads import WORKLOADS, Workload, make_workload
 
-    w = WORKLOADS[args.workload]
+    if args.custom:
+        cn, ckl, cku = args.custom[:3]
+        cb = args.custom[3] if len(args.custom) > 3 else 0
+        w = Workload(f"custom_n{cn}_kl{ckl}_ku{cku}" + (f"_batch{cb}" if cb else ""), cn, ckl, cku, "uniform",
+                     4.0 if cb else 0.0, 7, batch=cb)
+    else:
+        w = WORKLOADS[args.workload]
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     bandlu.load()
@@ -468,10 +519,14 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="workload name (default: the n=4096, kl=ku=16 matrix); others for per-workload reports")
+    ap.add_argument("--custom", type=int, nargs="+", metavar="N KL KU [BATCH]",
+                    help="per-stage report of a synthetic uniform[-1,1] band of this shape (batched if BATCH > 0)")
     args = ap.parse_args()
+    if args.custom is not None and len(args.custom) not in (3, 4):
+        ap.error("--custom takes N KL KU [BATCH]")
     if args.impl == "reference":
         run_reference(args)
-    elif args.workload != WORKLOAD:
+    elif args.custom or args.workload != WORKLOAD:
         run_workload_report(args)
     else:
         run_ours(args)
