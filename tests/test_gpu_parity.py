@@ -374,6 +374,21 @@ def test_batched_mixed_matrices():
     assert list(got["status"][6:8]) == [1, 1]
 
 
+def test_batched_many_small_varied_bands():
+    # more matrices than the persistent kernel has hand-off slots, bands from diagonal
+    # to wider than a register window, storage taller than the band (zeroed rows)
+    rng = np.random.default_rng(3)
+    n, ldab, batch = 40, 16, 2500
+    mats = []
+    for b in range(batch):
+        kl, ku = int(rng.integers(0, 5)), int(rng.integers(0, 6))
+        mats.append(banded(n, kl, ku, seed=b, boost=3.0 * float(rng.integers(0, 2))))
+    A = torch.stack(mats)
+    got = run_batched(A, ldab)
+    ref = oracle.dispatch_lu_batched(A.numpy(), ldab)
+    compare_batched(got, ref)
+
+
 @pytest.mark.parametrize("batch,n,kl,ku,lda", [(37, 256, 2, 2, 256), (16, 100, 3, 1, 101), (8, 1, 0, 0, 1),
                                                (5, 700, 10, 10, 700)])
 def test_batched_matches_oracle(batch, n, kl, ku, lda):
