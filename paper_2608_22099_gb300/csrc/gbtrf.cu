@@ -1,7 +1,8 @@
 // gbtrf.cu -- banded LU with partial pivoting (Sec. II-A step 3; f(N) ~ O(N*P*Q), Eq. S-N-N3).
 //
-// Two single-matrix kernels here (wide bands go first to the multi-CTA kernel
-// of gbtrf_wide.cu, when it can be launched):
+// Two single-matrix kernels here, after the narrowest bands (a one-warp
+// register window, k_gbtrf_regwin) and before the wide ones (the multi-CTA
+// kernel of gbtrf_wide.cu, when it can be launched):
 //
 //  * k_gbtrf_window (kl <= 27, the narrow bands the method targets).  One CTA.
 //    The active part of the band at step j is the dense (kl+1) x (kv+1) block
@@ -31,6 +32,7 @@
 
 #include "common.cuh"
 #include "rcp.cuh"
+#include "regwin.cuh"
 #include "sync.cuh"
 
 namespace bandlu {
@@ -428,6 +430,27 @@ __global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int
   if (tid == 0) *d_info = info;
 }
 
+// The narrowest bands, (kl+1)*(kl+ku+1) <= 32: one warp with the active window
+// in registers (regwin.cuh).  Fill-row entries above the matrix are cleared
+// first, as the elimination clears every fill row; the window writes the rest.
+__global__ void __launch_bounds__(32) k_gbtrf_regwin(int n, int kl, int ku, double *__restrict__ AB, int ldab,
+                                                     int *__restrict__ ipiv, int *__restrict__ d_info) {
+  const int kv = kl + ku, lane = threadIdx.x;
+  if (kl > 0) {
+    for (int e = lane; e < kl * min(n, kv); e += 32) {
+      const int jj = e / kl, rr = e - jj * kl;
+      if (rr < kv - jj) AB[rr + jj * ldab] = 0.0;
+    }
+  }
+  __syncwarp();
+  double *const abp[1] = {AB};
+  int *const pvp[1] = {ipiv};
+  const int klv[1] = {kl}, kuv[1] = {ku};
+  int info[1];
+  regwin::window_gbtrf<1>(abp, ldab, n, klv, kuv, pvp, info);
+  if (lane == 0) *d_info = info[0];
+}
+
 template <int K, int PF>
 int launch_window(long long n, int kl, int ku, double *AB, long long ldab, int *ipiv, int *d_info, size_t smem,
                   cudaStream_t s) {
@@ -461,6 +484,11 @@ int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv,
     return BANDLU_OK;
   }
   const long long kv = (long long)kl + ku;
+  if ((kl + 1LL) * (kv + 1) <= 32 && (n + 1) * ldab < (int64_t)INT_MAX) {
+    k_gbtrf_regwin<<<1, 32, 0, s>>>((int)n, kl, ku, AB, (int)ldab, ipiv, d_info);
+    BANDLU_CHECK_LAUNCH();
+    return BANDLU_OK;
+  }
   const long long CS = kl + kv + 1;
   const long long R = kl + 1 + kDelta;
   const size_t smem = (size_t)(R * CS) * sizeof(double);

@@ -165,12 +165,17 @@ def test_gbtrf_pivot_ties_take_the_first_row():
     assert_factor_parity(*gbtrf_gpu(AB, kl, ku), ref[0], ref[1], ref[2])
 
 
-def test_gbtrf_garbage_in_fill_rows_and_wider_storage():
-    n, kl, ku = 300, 6, 5
-    A = banded(n, kl, ku, seed=5).numpy()
-    AB = oracle.dense_to_band(A, kl, ku, ldab=2 * kl + ku + 1 + 3)
+@pytest.mark.parametrize("n,kl,ku", [(300, 6, 5), (300, 2, 3), (257, 0, 9), (200, 30, 12)])
+def test_gbtrf_garbage_in_fill_rows_and_wider_storage(n, kl, ku):
+    # fill rows hold garbage (the elimination clears them); rows beyond 2kl+ku hold
+    # garbage that no step may touch (the oracle leaves them as they are)
+    A = banded(n, kl, ku, seed=5 + kl).numpy()
+    ldab = 2 * kl + ku + 1 + 3
+    AB = oracle.dense_to_band(A, kl, ku, ldab=ldab)
     AB[:, :kl] = 321.0
+    AB[:, 2 * kl + ku + 1:] = -17.25
     ref = oracle.gbtrf(AB, kl, ku)
+    assert np.all(ref[0][:, 2 * kl + ku + 1:] == -17.25)
     assert_factor_parity(*gbtrf_gpu(AB, kl, ku), ref[0], ref[1], ref[2])
 
 
