@@ -4,17 +4,20 @@
 //
 // Columns are cut into blocks of kNB; block p is panel p.
 //
-//  * CTA 0 (panel CTA).  Nine compute warps own the rows of the current panel
-//    (thread i <-> row p*kNB + i, held in registers).  One panel step is one
-//    exact argmax round and ONE barrier: every warp publishes its best
+//  * CTA 0 (panel CTA).  Group A (nine warps) owns the rows of the current
+//    panel (thread i <-> row p*kNB + i, held in registers).  One panel step is
+//    one exact argmax round and ONE barrier: every warp publishes its best
 //    candidate together with that row's panel values, and the thread of row j
 //    publishes row j, so every thread can apply the interchange, form its
 //    multiplier and update its own row without further synchronisation.
-//    After panel p the compute warps apply panel p-1 and panel p to block p+1
-//    (a two-panel lookahead), which thereby becomes panel p+1.
-//    An I/O warp writes every finished panel block and its pivots to AB and
-//    ipiv, publishes them (panel_ready[p]), and prefetches block p+2 with
-//    cp.async once its owner has handed it over (block_ready[p+2]).
+//    After panel p group A applies panel p to block p+1, which thereby becomes
+//    panel p+1.  Group B (nine more warps) has meanwhile applied panel p-1 to
+//    block p+1, while group A factored panel p (a two-panel lookahead split
+//    over two warp groups, so that only one lookahead pass is on the serial
+//    path).  A storer warp writes every finished panel block and its pivots to
+//    AB and ipiv and publishes them (panel_ready[p]); a loader warp brings
+//    block b in with cp.async once its owner has handed it over
+//    (block_ready[b]) and its buffer is free.
 //  * CTAs 1..G (update CTAs) own the blocks b >= 3, block b on CTA
 //    1 + (b-3) mod G.  A block is read into shared memory when the first panel
 //    reaching it is published, receives panels p_first(b)..b-3 in order, and is
@@ -30,7 +33,8 @@
 // row-j entry are +0.0 fill, so this changes no bit.
 //
 // Hand-offs between CTAs are acquire/release flags in global memory, inside
-// the panel CTA mbarriers; every wait is bounded.  A wait that gives up raises
+// the panel CTA mbarrier rings (a ring of kRing entries per hand-off, deeper
+// than any producer can run ahead of its consumer); every wait is bounded.  A wait that gives up raises
 // an error flag that every waiter checks, the kernel ends, and *d_info becomes
 // -BANDLU_ERR_TIMEOUT.
 #include <climits>
@@ -44,14 +48,19 @@ namespace bandlu {
 namespace {
 
 constexpr int kNB = 4;                // panel width = column block width
-constexpr int kCW = 9;                // compute warps
-constexpr int kCT = 32 * kCW;         // compute threads
-constexpr int kThreads = kCT + 32;    // + the panel CTA's I/O warp
+constexpr int kCW = 9;                // warps of a compute group
+constexpr int kCT = 32 * kCW;         // threads of a compute group
+constexpr int kStoreWarp = 2 * kCW;   // panel CTA: group A = warps 0..8, group B = 9..17
+constexpr int kLoadWarp = kStoreWarp + 1;
+constexpr int kThreads = 32 * (kLoadWarp + 1);
+constexpr int kBarA = 1, kBarB = 2;   // named barriers of the two groups
+constexpr int kRing = 4;              // depth of the hand-off mbarrier rings
 constexpr int kMaxActive = 2;         // blocks an update CTA holds at once
 constexpr int kPanelBufs = 3;         // block buffers of the panel CTA
 constexpr long long kSpinLimit = 2000000000ll;
 
-__device__ __forceinline__ void bar_compute() { asm volatile("bar.sync 1, %0;" ::"n"(kCT) : "memory"); }
+__device__ __forceinline__ void bar_group(int id) { asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kCT) : "memory"); }
+__device__ __forceinline__ void bar_compute() { bar_group(kBarA); }
 
 __device__ __forceinline__ int ld_acquire(const int *p) {
   int v;
@@ -125,21 +134,31 @@ __device__ __forceinline__ bool handed_off(const Geo &g, int b) { return b >= 3 
 // Synchronisation and broadcast state.  Slots indexed [2] alternate with the
 // barrier count: a slot is rewritten only two barriers after it was published,
 // when every reader has passed the barrier in between.
+// Broadcast slots of one compute group's lookahead steps.
+struct Bcast {
+  double bu[2][kNB];   // pivot row in the block's columns
+  double br0[2][kNB];  // row j in the block's columns
+  unsigned bum[2];     // nonzero mask of bu
+};
+
 template <int RPT>
 struct WideShared {
   unsigned long long key[2][RPT * kCW];
   double piv[2][RPT * kCW][kNB];  // each warp's best candidate row, panel columns
   int idx[2][RPT * kCW];
   double row0[2][kNB];            // row j before the interchange, panel columns
-  double bu[2][kNB];              // lookahead: pivot row in the block's columns
-  double br0[2][kNB];             // lookahead: row j in the block's columns
-  unsigned bum[2];                // nonzero mask of bu
   unsigned pivm[2][RPT * kCW];    // nonzero masks of piv
+  Bcast bc[2];                    // group A, group B
   int pk[2][kNB];                 // pivot offsets of a panel, by panel parity
   int zp[2][kNB];                 // exact zero pivot
-  unsigned long long mb_done[2];  // compute -> I/O: panel p finished (mb_done[p & 1])
-  unsigned long long mb_load[2];  // I/O -> compute: block b in shared memory (mb_load[b & 1])
-  int ok;
+  int pvr[kRing][kNB];            // pivot offsets for the storer, by panel
+  // hand-off rings: entry i of a ring serves events i, i+kRing, ... (parity = which)
+  unsigned long long mb_done[kRing];    // A -> storer: panel p finished          (p)
+  unsigned long long mb_stored[kRing];  // storer -> loader: block p written out  (p)
+  unsigned long long mb_go[kRing];      // A -> B: panel b-2 finished            (b-2)
+  unsigned long long mb_loaded[kRing];  // loader -> B: block b in shared memory (b-2)
+  unsigned long long mb_bdone[kRing];   // B -> A: panel b-2 applied to block b  (b-2)
+  int ok[2];
   int info;
 };
 
@@ -163,14 +182,19 @@ __device__ __forceinline__ bool bounded_poll(F ready, int *err) {
   }
 }
 
-// All compute threads: thread 0 waits, the outcome is shared.
+// All threads of a compute group (tid = index in the group): its thread 0
+// waits, the outcome is shared.
+template <int RPT, class F>
+__device__ bool group_wait(F ready, int *err, WideShared<RPT> &sh, int tid, int grp) {
+  if (tid == 0) sh.ok[grp] = bounded_poll(ready, err) ? 1 : 0;
+  bar_group(grp == 0 ? kBarA : kBarB);
+  const bool ok = sh.ok[grp] != 0;
+  bar_group(grp == 0 ? kBarA : kBarB);
+  return ok;
+}
 template <int RPT, class F>
 __device__ bool compute_wait(F ready, int *err, WideShared<RPT> &sh) {
-  if (threadIdx.x == 0) sh.ok = bounded_poll(ready, err) ? 1 : 0;
-  bar_compute();
-  const bool ok = sh.ok != 0;
-  bar_compute();
-  return ok;
+  return group_wait<RPT>(ready, err, sh, threadIdx.x, 0);
 }
 
 // I/O warp: lane 0 waits, the outcome is warp-uniform.
@@ -217,6 +241,23 @@ __device__ void store_block(const Geo &g, double *AB, const double *blk, int b, 
   }
 }
 
+// Loader: one bulk (TMA) copy of a handed-off block of kNB full columns
+// (kNB * ldab * 8 bytes, a multiple of 16 with AB 16-byte aligned); it
+// completes the phase of *mbar once the bytes have landed.  The block was
+// written through ordinary stores by another CTA and acquired through its flag,
+// so the generic-to-async proxy fence comes first.
+__device__ void bulk_prefetch_block(const Geo &g, const double *AB, double *blk, int b, unsigned long long *mbar) {
+  const unsigned bytes = (unsigned)(kNB * g.ldab * sizeof(double));
+  const double *src = AB + (long long)b * kNB * g.ldab;
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(mbar)), "r"(bytes)
+               : "memory");
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_addr(blk)),
+               "l"(src), "r"(bytes), "r"(smem_addr(mbar))
+               : "memory");
+}
+
 // I/O warp: copy of a handed-off block in 16-byte cp.async chunks (AB aligned).
 __device__ void io_prefetch_block(const Geo &g, const double *AB, double *blk, int b) {
   const int lane = threadIdx.x & 31;
@@ -238,8 +279,7 @@ __device__ void io_prefetch_block(const Geo &g, const double *AB, double *blk, i
 // parity `bpar` advances at each barrier.
 template <int RPT>
 __device__ void apply_panel(const Geo &g, double *blk, int b, int q, const double (&lr)[RPT][kNB], const int *pk,
-                            const int *zp, WideShared<RPT> &sh, int &bpar) {
-  const int tid = threadIdx.x;
+                            const int *zp, Bcast &bc, int tid, int bar, int &bpar) {
   const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
   const int c0b = b * kNB, ncb = min(kNB, g.n - c0b);
   const int ldab = (int)g.ldab;
@@ -266,19 +306,19 @@ __device__ void apply_panel(const Geo &g, double *blk, int b, int q, const doubl
       const int i = tid + r * kCT;
       if (i == k + p) {
 #pragma unroll
-        for (int d = 0; d < kNB; ++d) sh.bu[s][d] = w[r][d];
-        sh.bum[s] = nz_mask(w[r]);
+        for (int d = 0; d < kNB; ++d) bc.bu[s][d] = w[r][d];
+        bc.bum[s] = nz_mask(w[r]);
       }
       if (i == k) {
 #pragma unroll
-        for (int d = 0; d < kNB; ++d) sh.br0[s][d] = w[r][d];
+        for (int d = 0; d < kNB; ++d) bc.br0[s][d] = w[r][d];
       }
     }
-    bar_compute();
+    bar_group(bar);
     double u[kNB];
 #pragma unroll
-    for (int d = 0; d < kNB; ++d) u[d] = sh.bu[s][d];
-    const unsigned um = sh.bum[s];
+    for (int d = 0; d < kNB; ++d) u[d] = bc.bu[s][d];
+    const unsigned um = bc.bum[s];
 #pragma unroll
     for (int r = 0; r < RPT; ++r) {
       const int i = tid + r * kCT;
@@ -287,7 +327,7 @@ __device__ void apply_panel(const Geo &g, double *blk, int b, int q, const doubl
         for (int d = 0; d < kNB; ++d) w[r][d] = u[d];
       } else if (p != 0 && i == k + p) {
 #pragma unroll
-        for (int d = 0; d < kNB; ++d) w[r][d] = sh.br0[s][d];
+        for (int d = 0; d < kNB; ++d) w[r][d] = bc.br0[s][d];
       }
       if (i > k && i <= k + km) {
         const double l = lr[r][k];
@@ -411,6 +451,23 @@ __device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, Wide
   }
 }
 
+// Multipliers of panel q for the rows of a compute group's threads (tid in the
+// group): lr[r][k] = l_{j+t, j}, j = q*kNB + k, t = tid + r*kCT - k.
+template <int RPT>
+__device__ __forceinline__ void panel_multipliers(const Geo &g, const double *ql, int q, int tid,
+                                                  double (&lr)[RPT][kNB]) {
+  const int c0q = q * kNB;
+#pragma unroll
+  for (int r = 0; r < RPT; ++r) {
+    const int i = tid + r * kCT;
+#pragma unroll
+    for (int k = 0; k < kNB; ++k) {
+      const int t = i - k;
+      lr[r][k] = (c0q + k < g.n && t >= 1 && t <= min(g.kl, g.n - 1 - (c0q + k))) ? ql[k * g.kl + t - 1] : 0.0;
+    }
+  }
+}
+
 template <int RPT>
 __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__restrict__ AB, int *__restrict__ ipiv,
                                                               int *__restrict__ d_info, int *__restrict__ flags) {
@@ -423,91 +480,125 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
   double *blocks = smem;                              // kPanelBufs (panel CTA) / kMaxActive blocks
   double *s_lbase = smem + (size_t)kPanelBufs * bsz;  // 2 panels of kNB * kl multipliers
   const int tid = threadIdx.x, warp = tid >> 5;
+  auto buf = [&](int b) { return blocks + (long long)(b % kPanelBufs) * bsz; };
+  auto mults = [&](int q) { return s_lbase + (size_t)(q & 1) * kNB * g.kl; };
+  auto ring_par = [](int e) { return (unsigned)(e / kRing) & 1u; };
 
   if (blockIdx.x == 0 && tid == 0) {
-    mbar_init(&sh.mb_done[0], 1);
-    mbar_init(&sh.mb_done[1], 1);
-    mbar_init(&sh.mb_load[0], 1);
-    mbar_init(&sh.mb_load[1], 1);
+    for (int i = 0; i < kRing; ++i) {
+      mbar_init(&sh.mb_done[i], 1);
+      mbar_init(&sh.mb_stored[i], 1);
+      mbar_init(&sh.mb_go[i], 1);
+      mbar_init(&sh.mb_loaded[i], 1);
+      mbar_init(&sh.mb_bdone[i], 1);
+    }
     sh.info = 0;
   }
   __syncthreads();
 
   if (blockIdx.x == 0) {
     if (warp < kCW) {
-      // ---------------- panel CTA: compute warps ----------------
+      // ---------------- panel CTA, group A: factorisation and lookahead of panel p ----------------
       int info = 0, bpar = 0;
-      load_block(g, AB, blocks, 0, true, tid, kCT);
-      if (g.npan > 1) load_block(g, AB, blocks + bsz, 1, true, tid, kCT);
+      load_block(g, AB, buf(0), 0, true, tid, kCT);
+      if (g.npan > 1) load_block(g, AB, buf(1), 1, true, tid, kCT);
       bar_compute();
       for (int p = 0; p < g.npan; ++p) {
-        double *cur = blocks + (long long)(p % kPanelBufs) * bsz;
-        double *s_l = s_lbase + (size_t)(p & 1) * kNB * g.kl;
-        factor_panel<RPT>(g, cur, p, s_l, sh, bpar, info);
-        if (tid == 0) sh.info = info;
+        factor_panel<RPT>(g, buf(p), p, mults(p), sh, bpar, info);
+        if (tid == 0) {
+          sh.info = info;
+#pragma unroll
+          for (int k = 0; k < kNB; ++k) sh.pvr[p % kRing][k] = sh.pk[p & 1][k];
+        }
         bar_compute();
-        if (tid == 0) mbar_arrive(&sh.mb_done[p & 1]);
+        if (tid == 0) {
+          mbar_arrive(&sh.mb_done[p % kRing]);
+          if (p + 2 < g.npan) mbar_arrive(&sh.mb_go[p % kRing]);  // B may apply panel p to block p+2
+        }
         if (p + 1 < g.npan) {
           const int b = p + 1;
-          double *nxt = blocks + (long long)(b % kPanelBufs) * bsz;
+          // block b holds panels <= b-2 (update CTAs and group B)
           if (b >= 2) {
-            unsigned long long *mb = &sh.mb_load[b & 1];
-            const unsigned par = (unsigned)((b - 2) >> 1) & 1u;
+            unsigned long long *mb = &sh.mb_bdone[(b - 2) % kRing];
+            const unsigned par = ring_par(b - 2);
             if (!compute_wait<RPT>([&] { return mbar_try_wait(mb, par); }, err, sh)) break;
           }
-          double lr[RPT][kNB];
-          for (int q = p - 1; q <= p; ++q) {
-            if (q < 0 || q < p_first(g, b)) continue;  // uniform
-            const double *ql = s_lbase + (size_t)(q & 1) * kNB * g.kl;
-            const int c0q = q * kNB;
-#pragma unroll
-            for (int r = 0; r < RPT; ++r) {
-              const int i = tid + r * kCT;
-#pragma unroll
-              for (int k = 0; k < kNB; ++k) {
-                const int t = i - k;
-                lr[r][k] = (c0q + k < g.n && t >= 1 && t <= min(g.kl, g.n - 1 - (c0q + k))) ? ql[k * g.kl + t - 1]
-                                                                                             : 0.0;
-              }
-            }
-            apply_panel<RPT>(g, nxt, b, q, lr, sh.pk[q & 1], sh.zp[q & 1], sh, bpar);
+          if (p >= p_first(g, b)) {  // uniform
+            double lr[RPT][kNB];
+            panel_multipliers<RPT>(g, mults(p), p, tid, lr);
+            apply_panel<RPT>(g, buf(b), b, p, lr, sh.pk[p & 1], sh.zp[p & 1], sh.bc[0], tid, kBarA, bpar);
             bar_compute();
           }
         }
       }
-    } else {
-      // ---------------- panel CTA: I/O warp ----------------
+    } else if (warp < kStoreWarp) {
+      // ---------------- panel CTA, group B: panel b-2 applied to block b ----------------
+      const int tidb = tid - kCT;
+      int bpar = 0;
+      for (int b = 2; b < g.npan; ++b) {
+        unsigned long long *mg = &sh.mb_go[(b - 2) % kRing];
+        unsigned long long *ml = &sh.mb_loaded[(b - 2) % kRing];
+        const unsigned par = ring_par(b - 2);
+        if (!group_wait<RPT>([&] { return mbar_try_wait(mg, par); }, err, sh, tidb, 1)) break;
+        if (!group_wait<RPT>([&] { return mbar_try_wait(ml, par); }, err, sh, tidb, 1)) break;
+        const int q = b - 2;
+        if (q >= p_first(g, b)) {  // uniform
+          double lr[RPT][kNB];
+          panel_multipliers<RPT>(g, mults(q), q, tidb, lr);
+          apply_panel<RPT>(g, buf(b), b, q, lr, sh.pk[q & 1], sh.zp[q & 1], sh.bc[1], tidb, kBarB, bpar);
+        }
+        bar_group(kBarB);
+        if (tidb == 0) mbar_arrive(&sh.mb_bdone[(b - 2) % kRing]);
+      }
+    } else if (warp == kStoreWarp) {
+      // ---------------- panel CTA, storer: finished panels to AB, published ----------------
       const int lane = tid & 31;
       for (int p = 0; p < g.npan; ++p) {
-        unsigned long long *mb = &sh.mb_done[p & 1];
-        const unsigned par = (unsigned)(p >> 1) & 1u;
+        unsigned long long *mb = &sh.mb_done[p % kRing];
+        const unsigned par = ring_par(p);
         if (!io_wait([&] { return mbar_try_wait(mb, par); }, err)) break;
         const int c0 = p * kNB, nc = min(kNB, g.n - c0);
-        store_block(g, AB, blocks + (long long)(p % kPanelBufs) * bsz, p, lane, 32);
-        if (lane < nc) ipiv[c0 + lane] = c0 + lane + sh.pk[p & 1][lane] + 1;
+        store_block(g, AB, buf(p), p, lane, 32);
+        if (lane < nc) ipiv[c0 + lane] = c0 + lane + sh.pvr[p % kRing][lane] + 1;
         __threadfence();
         __syncwarp();
-        if (lane == 0) st_release(panel_ready + p, 1);
-        const int b = p + 2;
-        if (b < g.npan) {
-          double *dst = blocks + (long long)(b % kPanelBufs) * bsz;
-          if (handed_off(g, b)) {
-            const int *f = block_ready + b;
-            if (!io_wait([&] { return ld_acquire(f) != 0; }, err)) break;
-            if (g.vec) {
-              io_prefetch_block(g, AB, dst, b);
-            } else {
-              load_block(g, AB, dst, b, false, lane, 32);
-            }
-          } else {
-            load_block(g, AB, dst, b, true, lane, 32);
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sh.mb_load[b & 1]);
+        if (lane == 0) {
+          st_release(panel_ready + p, 1);
+          mbar_arrive(&sh.mb_stored[p % kRing]);  // its buffer may take block p+3
         }
       }
       // info is final once the last panel is done; the status reflects every CTA's waits
       if (lane == 0) *d_info = ld_acquire(err) ? -BANDLU_ERR_TIMEOUT : sh.info;
+    } else {
+      // ---------------- panel CTA, loader: blocks b >= 2 into shared memory ----------------
+      const int lane = tid & 31;
+      for (int b = 2; b < g.npan; ++b) {
+        if (b >= 3) {  // the buffer held block b-3
+          unsigned long long *mb = &sh.mb_stored[(b - 3) % kRing];
+          const unsigned par = ring_par(b - 3);
+          if (!io_wait([&] { return mbar_try_wait(mb, par); }, err)) break;
+        }
+        double *dst = buf(b);
+        unsigned long long *ml = &sh.mb_loaded[(b - 2) % kRing];
+        if (handed_off(g, b)) {
+          const int *f = block_ready + b;
+          if (!io_wait([&] { return ld_acquire(f) != 0; }, err)) break;
+          if (g.vec && (b + 1) * kNB <= g.n) {
+            if (lane == 0) bulk_prefetch_block(g, AB, dst, b, ml);  // completes the phase itself
+            __syncwarp();
+            continue;
+          }
+          if (g.vec) {
+            io_prefetch_block(g, AB, dst, b);
+          } else {
+            load_block(g, AB, dst, b, false, lane, 32);
+          }
+        } else {
+          load_block(g, AB, dst, b, true, lane, 32);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(ml);
+      }
     }
   } else {
     // ---------------- update CTAs ----------------
@@ -546,7 +637,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
           load_block(g, AB, blk, b, true, tid, kCT);
           bar_compute();
         }
-        apply_panel<RPT>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh, bpar);
+        apply_panel<RPT>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh.bc[0], tid, kBarA, bpar);
         bar_compute();
         if (p == b - 3) {
           store_block(g, AB, blk, b, tid, kCT);
