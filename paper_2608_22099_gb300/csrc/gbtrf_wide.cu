@@ -148,6 +148,8 @@ struct WideShared {
   int idx[2][RPT * kCW];
   double row0[2][kNB];            // row j before the interchange, panel columns
   unsigned pivm[2][RPT * kCW];    // nonzero masks of piv
+  double prc[2][RPT * kCW];       // correctly rounded reciprocal of each partial's candidate
+  int pspec[2][RPT * kCW];        // ... not formed (zero, subnormal, huge, inf, nan)
   Bcast bc[2];                    // group A, group B
   int pk[2][kNB];                 // pivot offsets of a panel, by panel parity
   int zp[2][kNB];                 // exact zero pivot
@@ -377,6 +379,9 @@ __device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, Wide
 #pragma unroll
     for (int r = 0; r < RPT; ++r) {
       const int i = tid + r * kCT, t = i - k;
+      // every thread forms the reciprocal of its own candidate while the argmax runs
+      bool myspec;
+      const double myr = rcp_rn_fast(v[r][k], &myspec);
       const unsigned long long key = (t >= 0 && t <= km) ? pivot_key(v[r][k], t == 0) : 0ull;
       unsigned long long kmax;
       const int wl = warp_first_max(key, &kmax);
@@ -386,6 +391,8 @@ __device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, Wide
 #pragma unroll
         for (int d = 0; d < kNB; ++d) sh.piv[s][r * kCW + warp][d] = v[r][d];
         sh.pivm[s][r * kCW + warp] = nz_mask(v[r]);
+        sh.prc[s][r * kCW + warp] = myr;
+        sh.pspec[s][r * kCW + warp] = myspec ? 1 : 0;
       }
       if (i == k) {
 #pragma unroll
@@ -416,7 +423,8 @@ __device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, Wide
       if (zero && info == 0) info = j + 1;
     }
     if (!zero) {
-      const double rc = rcp_rn(u[k]);
+      double rc = sh.prc[s][wb];
+      if (sh.pspec[s][wb]) rc = rcp_division(u[k]);  // uniform
 #pragma unroll
       for (int r = 0; r < RPT; ++r) {
         const int i = tid + r * kCT;
@@ -558,14 +566,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
         const unsigned par = ring_par(p);
         if (!io_wait([&] { return mbar_try_wait(mb, par); }, err)) break;
         const int c0 = p * kNB, nc = min(kNB, g.n - c0);
-        store_block(g, AB, buf(p), p, lane, 32);
+        const double *src = buf(p);
+        double *dst = AB + (long long)c0 * g.ldab;
+        const int ld = (int)g.ldab;
+        // what the update CTAs read first: the diagonal and the multipliers (rows
+        // kv..kv+kl of the panel's columns) and the pivots; then the publication
+        for (int k = 0; k < nc; ++k)
+          for (int rr = g.kv + lane; rr <= g.kv + g.kl; rr += 32) dst[k * ld + rr] = src[k * ld + rr];
         if (lane < nc) ipiv[c0 + lane] = c0 + lane + sh.pvr[p % kRing][lane] + 1;
         __threadfence();
         __syncwarp();
-        if (lane == 0) {
-          st_release(panel_ready + p, 1);
-          mbar_arrive(&sh.mb_stored[p % kRing]);  // its buffer may take block p+3
-        }
+        if (lane == 0) st_release(panel_ready + p, 1);
+        // then the whole block (the published rows again, unchanged)
+        store_block(g, AB, src, p, lane, 32);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh.mb_stored[p % kRing]);  // its buffer may take block p+3
       }
       // info is final once the last panel is done; the status reflects every CTA's waits
       if (lane == 0) *d_info = ld_acquire(err) ? -BANDLU_ERR_TIMEOUT : sh.info;
