@@ -224,12 +224,10 @@ def run_ours(args):
     import torch
     import torch.distributed as dist
 
-    from paper_2608_22099_gb300 import bandlu
+    from paper_2608_22099_gb300 import bandlu, multirank
     from paper_2608_22099_gb300.workloads import WORKLOADS, make_workload
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    rank, world, local = multirank.rank_info()
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     if world > 1:
@@ -281,11 +279,9 @@ def run_ours(args):
     barrier()
     t_wall1 = time.time()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    total_ms = torch.tensor([sum(step_ms)], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(total_ms, op=dist.ReduceOp.MAX)
-    ms_per_step = float(total_ms.item()) / args.steps
-    value = world * flops / (ms_per_step * 1e-3) / 1e9
+    # replicas: every rank factors its own matrix; the job's time is the slowest rank's
+    ms_per_step = multirank.max_over_ranks(sum(step_ms), device=dev) / args.steps
+    value = multirank.job_throughput(multirank.sum_over_ranks(flops, device=dev), ms_per_step * 1e-3) / 1e9
 
     # stage breakdown through the same C ABI, CUDA events on the launching stream
     klku = torch.zeros(2, dtype=torch.int32, device=dev)
@@ -362,11 +358,8 @@ def run_ours(args):
         info_host.copy_(info, non_blocking=True)
         e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
-    e2e_t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(e2e_t, op=dist.ReduceOp.MAX)
-    e2e_value = world * flops / (float(e2e_t.item()) * 1e-3) / 1e9
+    e2e_ms = multirank.max_over_ranks(statistics.mean(a.elapsed_time(b) for a, b in e2e_ev), device=dev)
+    e2e_value = multirank.job_throughput(multirank.sum_over_ranks(flops, device=dev), e2e_ms * 1e-3) / 1e9
     h2d = A_host.numel() * 8
     d2h = AB_host.numel() * 8 + ipiv_host.numel() * 4 + info_host.numel() * 4
 
@@ -399,7 +392,7 @@ def run_ours(args):
             "flops_per_step": flops, "stages": stages, "roofline": roofline,
             "cpu_baseline": cpu_baseline,
             "e2e": {"value": e2e_value, "unit": "GFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "ms_per_step": float(e2e_t.item())},
+                    "ms_per_step": e2e_ms},
             "gpu_launches": 3 * args.steps,
             "clocks": clocks,
             "wall_s_timed": t_wall1 - t_wall0,
