@@ -41,7 +41,7 @@ FALLBACK_HBM_GBS = 6800.0
 # Sources of each kernel: a DRAM-traffic figure taken by ncu is valid only while
 # their hash is the one recorded beside it under profiles/.
 KERNEL_SOURCES = {
-    "k_gbtrf_window": ["gbtrf.cu", "common.cuh", "rcp.cuh", "sync.cuh"],
+    "k_gbtrf_window": ["gbtrf.cu", "common.cuh", "rcp.cuh", "sync.cuh", "regwin.cuh"],
     "k_detect_vec": ["detect.cu", "common.cuh"],
     "k_dense_to_band_tiled": ["convert.cu", "common.cuh"],
 }
