@@ -77,6 +77,20 @@ def profiled_traffic(kernel: str):
     return None
 
 
+class L2Flush:
+    """Cold L2 before a timed call: a 512 MiB write (larger than the 126 MiB L2), then a
+    256 MiB read of another buffer, which writes the flush's dirty lines back to HBM before the
+    call instead of during it.  Both run on the stream outside the timed events."""
+
+    def __init__(self, torch, dev):
+        self.w = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)
+        self.r = torch.zeros(256 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)
+
+    def __call__(self, k: int = 0):
+        self.w.fill_(k)
+        self.r.max()
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -244,7 +258,7 @@ def run_ours(args):
     AB = torch.zeros((n, ldab), dtype=torch.float64, device=dev)
     ipiv = torch.zeros(n, dtype=torch.int32, device=dev)
     info = torch.zeros(1, dtype=torch.int32, device=dev)
-    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)  # 512 MiB > L2 (126 MiB)
+    flush = L2Flush(torch, dev)
     stream = torch.cuda.current_stream()
 
     def step():
@@ -253,7 +267,7 @@ def run_ours(args):
             raise RuntimeError(f"dispatch_lu returned {rc} ({gkl}, {gku})")
 
     for _ in range(max(args.warmup, 3)):
-        flush.fill_(1)
+        flush(1)
         step()
     torch.cuda.synchronize()
     if int(info.item()) != 0:
@@ -271,7 +285,7 @@ def run_ours(args):
     torch.cuda.synchronize()
     t_wall0 = time.time()
     for k in range(args.steps):
-        flush.fill_(k)                 # L2 flush between steps, outside the timed events
+        flush(k)                       # L2 flush between steps, outside the timed events
         starts[k].record(stream)
         step()
         ends[k].record(stream)
@@ -291,7 +305,7 @@ def run_ours(args):
     reps = min(args.steps, 50)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(reps)]
     for r in range(reps):
-        flush.fill_(r)
+        flush(r)
         e = ev[r]
         e[0].record(stream)
         bandlu.check(bandlu.detect_bandwidth(A, n, n, klku, klku.data_ptr() + 4, stream), "detect_bandwidth")
@@ -347,7 +361,7 @@ def run_ours(args):
     e2e_reps = min(args.steps, 50)
     e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(e2e_reps)]
     for r in range(e2e_reps):
-        flush.fill_(r)
+        flush(r)
         e0, e1 = e2e_ev[r]
         e0.record(stream)
         A_e2e.copy_(A_host, non_blocking=True)
@@ -385,7 +399,7 @@ def run_ours(args):
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": WORKLOAD, "n": n, "kl": kl, "ku": ku, "ldab": ldab, "dist": "uniform[-1,1]",
-                       "l2": "flushed between steps (512 MiB write)",
+                       "l2": "flushed between steps (512 MiB write, then a 256 MiB read that writes its dirty lines back)",
                        "parallelism": "replicas" if world > 1 else "single"},
             "dispatch_ms": ms_per_step, "dense_lu_ms": dense_t,
             "speedup_over_dense": (dense_t / ms_per_step) if dense_t else None,
@@ -422,7 +436,7 @@ def run_workload_report(args):
     bandlu.load()
     A = make_workload(w, device=dev)
     n, kl, ku, ldab = w.n, w.kl, w.ku, w.ldab
-    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)
+    flush = L2Flush(torch, dev)
     stream = torch.cuda.current_stream()
     hbm_peak, hbm_src = load_peaks()
     out = {"workload": w.name, "n": n, "kl": kl, "ku": ku, "batch": w.batch}
@@ -431,7 +445,7 @@ def run_workload_report(args):
     def timed(fn, reps):
         ts = []
         for r in range(reps):
-            flush.fill_(r)
+            flush(r)
             a = torch.cuda.Event(enable_timing=True); b = torch.cuda.Event(enable_timing=True)
             a.record(stream)
             fn()
