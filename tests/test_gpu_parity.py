@@ -232,6 +232,18 @@ def test_gbtrf_wide_blocks_share_update_ctas():
     assert_factor_parity(*gbtrf_gpu(AB, kl, ku), ref[0], ref[1], ref[2])
 
 
+@pytest.mark.parametrize("n,kl,ku", [(701, 600, 10), (613, 290, 33)])
+def test_gbtrf_wide_several_rows_per_thread(n, kl, ku):
+    # kl + 4 panel rows exceed one compute group's 288 threads: 2 (kl = 290) and 3-4 (kl = 600)
+    # rows per thread
+    A = banded(n, kl, ku, seed=n + kl, dist="normal").numpy()
+    AB = oracle.dense_to_band(A, kl, ku)
+    ref = oracle.gbtrf(AB, kl, ku)
+    got = gbtrf_gpu(AB, kl, ku)
+    assert_factor_parity(*got, ref[0], ref[1], ref[2])
+    assert oracle.backward_error(A, got[0], got[1], kl, ku) <= 10.0
+
+
 def test_gbtrf_wide_zero_pivots_garbage_fill_and_wider_storage():
     n, kl, ku = 500, 40, 31
     A = banded(n, kl, ku, seed=23).numpy()
