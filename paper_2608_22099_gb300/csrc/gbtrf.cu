@@ -300,21 +300,36 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
     }
   } else if ((warp & 3) != 0) {
     // ---------------- updater warps: columns j+3 .. j+kv ----------------
-    const int uw = warp - 1 - (warp >> 2) - (warp > kIoWarp ? 1 : 0);  // 0..kNU-1
+    // Updater index of this warp.  The order puts the warps that also take the
+    // last, partial round of elements on different SMSPs, so that the FP64
+    // instructions of a step spread evenly over the SMSPs' pipes.
+    constexpr int kUw[16] = {-1, 0, 2, 3, -1, 1, 4, 5, -1, 6, 7, 8, -1, -1, 9, 10};
+    const int uw = kUw[warp];  // 0..kNU-1
     const int tid_u = uw * 32 + lane;
     const int ncols = kv > 2 ? kv - 2 : 0;
     const int E = ncols * (kl + 1);
-    // Static element map, columns fastest: element e -> row offset t = e / ncols
-    // (t = 0: the U row is written out), column offset d = 3 + e % ncols.  The
-    // lanes of a warp then read one row record (a broadcast) and consecutive
-    // columns of the pivot row and of their own row (no bank conflicts).
+    const int EF = ncols * kl;  // elements with a multiply-add (rows t >= 1)
+    // Static element map, columns fastest: elements 0..EF-1 are row offsets
+    // t = 1 + e / ncols, column offsets d = 3 + e % ncols; the last ncols
+    // elements are the U row (t = 0), which is only written out.  The lanes of
+    // a warp read one row record (a broadcast) and consecutive columns of the
+    // pivot row and of their own row (no bank conflicts), and every warp
+    // instruction of the multiply-adds is full except the last.
     int ed[K], et[K];
     long long uoff[K];  // offset of U(j, j+d) in AB relative to column j
 #pragma unroll
     for (int k = 0; k < K; ++k) {
       const int e = tid_u + kNUT * k;
-      et[k] = e < E ? e / ncols : 0;
-      ed[k] = e < E ? 3 + (e - et[k] * ncols) : 0;
+      if (e < EF) {
+        et[k] = 1 + e / ncols;
+        ed[k] = 3 + (e - (et[k] - 1) * ncols);
+      } else if (e < E) {
+        et[k] = 0;
+        ed[k] = 3 + (e - EF);
+      } else {
+        et[k] = 0;
+        ed[k] = 0;
+      }
       uoff[k] = (kv - ed[k]) + (long long)ed[k] * ldab;
     }
     int qj = 0;  // column slot of column j
