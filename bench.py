@@ -13,6 +13,7 @@ data-parallel split), one per GPU.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
   python bench.py --workload NAME [--steps K]     per-stage report of a named workload
   python bench.py --custom N KL KU [BATCH]        the same report for a synthetic shape
+  python bench.py --sweep                         the paper's experiments A-C on this GPU
 """
 from __future__ import annotations
 
@@ -533,6 +534,74 @@ def run_workload_report(args):
     print(json.dumps(out), flush=True)
 
 
+def run_sweep(args):
+    """The paper's experiments on this GPU (Sec. IV): A, the speedup of dispatch_lu over the
+    dense LU for N = 2000..8000 with P + Q = 1% and 10% of N (Eq. su-con; Sec. III-C predicts
+    linear growth in N); B, the slowdown (I + F) / F on the same shapes with one stray entry
+    that makes them non-banded (Eq. sd-con; predicted constant); C, the N = 10^4, 100 + 100
+    diagonals case of Figs. 5-6, with the memory ratio.  One JSON line per point."""
+    import torch
+
+    from paper_2608_22099_gb300 import bandlu
+    from paper_2608_22099_gb300.workloads import make_dense
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    bandlu.load()
+    flush = L2Flush(torch, dev)
+    stream = torch.cuda.current_stream()
+    reps = max(1, min(args.steps, 5))
+
+    def timed(fn):
+        ts = []
+        for r in range(reps):
+            flush(r)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b) * 1e-3)
+        return statistics.median(ts)
+
+    points = [("A", n, f) for f in (0.01, 0.10) for n in range(2000, 8001, 1000)] + [("C", 10000, 0.02)]
+    for exp, n, f in points:
+        kl = ku = max(1, int(round(f * n / 2)))
+        ldab = 2 * kl + ku + 1
+        A = make_dense(n, kl, ku, dist="uniform", seed=n + kl, device=dev)
+        AB = torch.zeros((n, ldab), dtype=torch.float64, device=dev)
+        ipiv = torch.zeros(n, dtype=torch.int32, device=dev)
+        info = torch.zeros(1, dtype=torch.int32, device=dev)
+        res = {}
+
+        def disp():
+            res["rc"] = bandlu.dispatch_lu(A, n, n, AB, ldab, ipiv, info, stream)
+
+        disp()
+        torch.cuda.synchronize()
+        t_disp = timed(disp)
+        t_dense = dense_lu_ms(torch, A, stream)
+        line = {"sweep": exp, "n": n, "kl": kl, "ku": ku, "p_plus_q_frac": (kl + ku) / n,
+                "status": res["rc"][0], "dispatch_ms": t_disp * 1e3, "dense_lu_ms": t_dense,
+                "speedup_over_dense": (t_dense * 1e-3 / t_disp) if t_dense else None,
+                "memory_ratio_dense_over_band": (8.0 * n * n + 8 * n) / (3 * 8.0 * ldab * n + 8 * n)}
+        # experiment B: the same shape with one stray entry -> not banded, detection + dense LU
+        A[n - 1, 0] = 1e-3
+        klku = torch.zeros(2, dtype=torch.int32, device=dev)
+
+        def det():
+            bandlu.check(bandlu.detect_bandwidth(A, n, n, klku, klku.data_ptr() + 4, stream), "detect")
+
+        rc_c, _, _ = bandlu.dispatch_lu(A, n, n, AB, ldab, ipiv, info, stream)
+        t_det = timed(det)
+        if t_dense:
+            line.update({"control_status": rc_c, "detect_us": t_det * 1e6,
+                         "slowdown_control": (t_det + t_dense * 1e-3) / (t_dense * 1e-3)})
+        print(json.dumps(line), flush=True)
+        del A, AB
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -542,6 +611,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="workload name (default: the n=4096, kl=ku=16 matrix); others for per-workload reports")
+    ap.add_argument("--sweep", action="store_true", help="the paper's experiments A-C (speedup / slowdown in N)")
     ap.add_argument("--custom", type=int, nargs="+", metavar="N KL KU [BATCH]",
                     help="per-stage report of a synthetic uniform[-1,1] band of this shape (batched if BATCH > 0)")
     args = ap.parse_args()
@@ -549,6 +619,8 @@ def main():
         ap.error("--custom takes N KL KU [BATCH]")
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep:
+        run_sweep(args)
     elif args.custom or args.workload != WORKLOAD:
         run_workload_report(args)
     else:
