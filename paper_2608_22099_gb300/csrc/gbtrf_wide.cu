@@ -48,19 +48,28 @@ namespace bandlu {
 namespace {
 
 constexpr int kNB = 4;                // panel width = column block width
-constexpr int kCW = 9;                // warps of a compute group
-constexpr int kCT = 32 * kCW;         // threads of a compute group
-constexpr int kStoreWarp = 2 * kCW;   // panel CTA: group A = warps 0..8, group B = 9..17
-constexpr int kLoadWarp = kStoreWarp + 1;
-constexpr int kThreads = 32 * (kLoadWarp + 1);
+// A compute group has CW warps (a template parameter: 2, 4 or 9, the fewest that
+// give every row of a panel, kl + kNB of them, its own thread).  The panel CTA
+// runs two groups (A: warps 0..CW-1, B: CW..2CW-1), a storer and a loader warp.
+template <int CW>
+struct Lay {
+  static constexpr int kCT = 32 * CW;            // threads of a compute group
+  static constexpr int kStoreWarp = 2 * CW;
+  static constexpr int kLoadWarp = kStoreWarp + 1;
+  static constexpr int kThreads = 32 * (kLoadWarp + 1);
+};
 constexpr int kBarA = 1, kBarB = 2;   // named barriers of the two groups
 constexpr int kRing = 4;              // depth of the hand-off mbarrier rings
 constexpr int kMaxActive = 2;         // blocks an update CTA holds at once
 constexpr int kPanelBufs = 3;         // block buffers of the panel CTA
 constexpr long long kSpinLimit = 2000000000ll;
 
-__device__ __forceinline__ void bar_group(int id) { asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kCT) : "memory"); }
-__device__ __forceinline__ void bar_compute() { bar_group(kBarA); }
+template <int CW>
+__device__ __forceinline__ void bar_group(int id) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(Lay<CW>::kCT) : "memory");
+}
+template <int CW>
+__device__ __forceinline__ void bar_compute() { bar_group<CW>(kBarA); }
 
 __device__ __forceinline__ int ld_acquire(const int *p) {
   int v;
@@ -141,8 +150,9 @@ struct Bcast {
   unsigned bum[2];     // nonzero mask of bu
 };
 
-template <int RPT>
+template <int CW, int RPT>
 struct WideShared {
+  static constexpr int kCW = CW;
   unsigned long long key[2][RPT * kCW];
   double piv[2][RPT * kCW][kNB];  // each warp's best candidate row, panel columns
   int idx[2][RPT * kCW];
@@ -186,17 +196,17 @@ __device__ __forceinline__ bool bounded_poll(F ready, int *err) {
 
 // All threads of a compute group (tid = index in the group): its thread 0
 // waits, the outcome is shared.
-template <int RPT, class F>
-__device__ bool group_wait(F ready, int *err, WideShared<RPT> &sh, int tid, int grp) {
+template <int CW, int RPT, class F>
+__device__ bool group_wait(F ready, int *err, WideShared<CW, RPT> &sh, int tid, int grp) {
   if (tid == 0) sh.ok[grp] = bounded_poll(ready, err) ? 1 : 0;
-  bar_group(grp == 0 ? kBarA : kBarB);
+  bar_group<CW>(grp == 0 ? kBarA : kBarB);
   const bool ok = sh.ok[grp] != 0;
-  bar_group(grp == 0 ? kBarA : kBarB);
+  bar_group<CW>(grp == 0 ? kBarA : kBarB);
   return ok;
 }
-template <int RPT, class F>
-__device__ bool compute_wait(F ready, int *err, WideShared<RPT> &sh) {
-  return group_wait<RPT>(ready, err, sh, threadIdx.x, 0);
+template <int CW, int RPT, class F>
+__device__ bool compute_wait(F ready, int *err, WideShared<CW, RPT> &sh) {
+  return group_wait<CW, RPT>(ready, err, sh, threadIdx.x, 0);
 }
 
 // I/O warp: lane 0 waits, the outcome is warp-uniform.
@@ -279,9 +289,10 @@ __device__ void io_prefetch_block(const Geo &g, const double *AB, double *blk, i
 // Compute threads; thread i <-> row q*kNB + i (the rows of panel q's steps).
 // lr[r][k]: multiplier of the thread's row r at step k (0 if none).  The slot
 // parity `bpar` advances at each barrier.
-template <int RPT>
+template <int CW, int RPT>
 __device__ void apply_panel(const Geo &g, double *blk, int b, int q, const double (&lr)[RPT][kNB], const int *pk,
                             const int *zp, Bcast &bc, int tid, int bar, int &bpar) {
+  constexpr int kCT = Lay<CW>::kCT;
   const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
   const int c0b = b * kNB, ncb = min(kNB, g.n - c0b);
   const int ldab = (int)g.ldab;
@@ -316,7 +327,7 @@ __device__ void apply_panel(const Geo &g, double *blk, int b, int q, const doubl
         for (int d = 0; d < kNB; ++d) bc.br0[s][d] = w[r][d];
       }
     }
-    bar_group(bar);
+    bar_group<CW>(bar);
     double u[kNB];
 #pragma unroll
     for (int d = 0; d < kNB; ++d) u[d] = bc.bu[s][d];
@@ -353,9 +364,10 @@ __device__ void apply_panel(const Geo &g, double *blk, int b, int q, const doubl
 // Factors block p in place; records the pivot offsets and zero flags in
 // sh.pk/sh.zp[p & 1] and the multipliers in s_l (s_l[k*kl + t-1] = l_{j+t, j},
 // j = p*kNB + k).
-template <int RPT>
-__device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, WideShared<RPT> &sh, int &bpar,
+template <int CW, int RPT>
+__device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, WideShared<CW, RPT> &sh, int &bpar,
                              int &info) {
+  constexpr int kCT = Lay<CW>::kCT, kCW = CW;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int c0 = p * kNB, nc = min(kNB, g.n - c0);
   const int ldab = (int)g.ldab;
@@ -399,7 +411,7 @@ __device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, Wide
         for (int d = 0; d < kNB; ++d) sh.row0[s][d] = v[r][d];
       }
     }
-    bar_compute();
+    bar_compute<CW>();
     // the first largest key over the partials, which are in row order
     unsigned long long best = sh.key[s][0];
     int wb = 0;
@@ -461,9 +473,10 @@ __device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, Wide
 
 // Multipliers of panel q for the rows of a compute group's threads (tid in the
 // group): lr[r][k] = l_{j+t, j}, j = q*kNB + k, t = tid + r*kCT - k.
-template <int RPT>
+template <int CW, int RPT>
 __device__ __forceinline__ void panel_multipliers(const Geo &g, const double *ql, int q, int tid,
                                                   double (&lr)[RPT][kNB]) {
+  constexpr int kCT = Lay<CW>::kCT;
   const int c0q = q * kNB;
 #pragma unroll
   for (int r = 0; r < RPT; ++r) {
@@ -476,11 +489,13 @@ __device__ __forceinline__ void panel_multipliers(const Geo &g, const double *ql
   }
 }
 
-template <int RPT>
-__global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__restrict__ AB, int *__restrict__ ipiv,
-                                                              int *__restrict__ d_info, int *__restrict__ flags) {
+template <int CW, int RPT>
+__global__ void __launch_bounds__(Lay<CW>::kThreads, 1)
+    k_gbtrf_wide(Geo g, double *__restrict__ AB, int *__restrict__ ipiv, int *__restrict__ d_info,
+                 int *__restrict__ flags) {
+  constexpr int kCT = Lay<CW>::kCT, kCW = CW, kStoreWarp = Lay<CW>::kStoreWarp;
   extern __shared__ __align__(16) double smem[];
-  __shared__ WideShared<RPT> sh;
+  __shared__ WideShared<CW, RPT> sh;
   int *err = flags;
   int *panel_ready = flags + 2;
   int *block_ready = flags + 2 + g.npan;
@@ -510,15 +525,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
       int info = 0, bpar = 0;
       load_block(g, AB, buf(0), 0, true, tid, kCT);
       if (g.npan > 1) load_block(g, AB, buf(1), 1, true, tid, kCT);
-      bar_compute();
+      bar_compute<CW>();
       for (int p = 0; p < g.npan; ++p) {
-        factor_panel<RPT>(g, buf(p), p, mults(p), sh, bpar, info);
+        factor_panel<CW, RPT>(g, buf(p), p, mults(p), sh, bpar, info);
         if (tid == 0) {
           sh.info = info;
 #pragma unroll
           for (int k = 0; k < kNB; ++k) sh.pvr[p % kRing][k] = sh.pk[p & 1][k];
         }
-        bar_compute();
+        bar_compute<CW>();
         if (tid == 0) {
           mbar_arrive(&sh.mb_done[p % kRing]);
           if (p + 2 < g.npan) mbar_arrive(&sh.mb_go[p % kRing]);  // B may apply panel p to block p+2
@@ -529,13 +544,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
           if (b >= 2) {
             unsigned long long *mb = &sh.mb_bdone[(b - 2) % kRing];
             const unsigned par = ring_par(b - 2);
-            if (!compute_wait<RPT>([&] { return mbar_try_wait(mb, par); }, err, sh)) break;
+            if (!compute_wait<CW, RPT>([&] { return mbar_try_wait(mb, par); }, err, sh)) break;
           }
           if (p >= p_first(g, b)) {  // uniform
             double lr[RPT][kNB];
-            panel_multipliers<RPT>(g, mults(p), p, tid, lr);
-            apply_panel<RPT>(g, buf(b), b, p, lr, sh.pk[p & 1], sh.zp[p & 1], sh.bc[0], tid, kBarA, bpar);
-            bar_compute();
+            panel_multipliers<CW, RPT>(g, mults(p), p, tid, lr);
+            apply_panel<CW, RPT>(g, buf(b), b, p, lr, sh.pk[p & 1], sh.zp[p & 1], sh.bc[0], tid, kBarA, bpar);
+            bar_compute<CW>();
           }
         }
       }
@@ -547,15 +562,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
         unsigned long long *mg = &sh.mb_go[(b - 2) % kRing];
         unsigned long long *ml = &sh.mb_loaded[(b - 2) % kRing];
         const unsigned par = ring_par(b - 2);
-        if (!group_wait<RPT>([&] { return mbar_try_wait(mg, par); }, err, sh, tidb, 1)) break;
-        if (!group_wait<RPT>([&] { return mbar_try_wait(ml, par); }, err, sh, tidb, 1)) break;
+        if (!group_wait<CW, RPT>([&] { return mbar_try_wait(mg, par); }, err, sh, tidb, 1)) break;
+        if (!group_wait<CW, RPT>([&] { return mbar_try_wait(ml, par); }, err, sh, tidb, 1)) break;
         const int q = b - 2;
         if (q >= p_first(g, b)) {  // uniform
           double lr[RPT][kNB];
-          panel_multipliers<RPT>(g, mults(q), q, tidb, lr);
-          apply_panel<RPT>(g, buf(b), b, q, lr, sh.pk[q & 1], sh.zp[q & 1], sh.bc[1], tidb, kBarB, bpar);
+          panel_multipliers<CW, RPT>(g, mults(q), q, tidb, lr);
+          apply_panel<CW, RPT>(g, buf(b), b, q, lr, sh.pk[q & 1], sh.zp[q & 1], sh.bc[1], tidb, kBarB, bpar);
         }
-        bar_group(kBarB);
+        bar_group<CW>(kBarB);
         if (tidb == 0) mbar_arrive(&sh.mb_bdone[(b - 2) % kRing]);
       }
     } else if (warp == kStoreWarp) {
@@ -626,7 +641,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
       const int b0 = lo + ((u - (lo - 3)) % G + G) % G;
       if (b0 > hi) continue;
       const int *f = panel_ready + p;
-      if (!compute_wait<RPT>([&] { return ld_acquire(f) != 0; }, err, sh)) break;
+      if (!compute_wait<CW, RPT>([&] { return ld_acquire(f) != 0; }, err, sh)) break;
       const int c0q = p * kNB, ncq = min(kNB, g.n - c0q);
       if (tid < kNB) {
         const int k = tid;
@@ -645,19 +660,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
                          : 0.0;
         }
       }
-      bar_compute();
+      bar_compute<CW>();
       for (int b = b0; b <= hi; b += G) {
         double *blk = blocks + (long long)(((b - 3) / G) % kMaxActive) * bsz;
         if (p == p_first(g, b)) {
           load_block(g, AB, blk, b, true, tid, kCT);
-          bar_compute();
+          bar_compute<CW>();
         }
-        apply_panel<RPT>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh.bc[0], tid, kBarA, bpar);
-        bar_compute();
+        apply_panel<CW, RPT>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh.bc[0], tid, kBarA, bpar);
+        bar_compute<CW>();
         if (p == b - 3) {
           store_block(g, AB, blk, b, tid, kCT);
           __threadfence();
-          bar_compute();
+          bar_compute<CW>();
           if (tid == 0) st_release(block_ready + b, 1);
         }
       }
@@ -667,22 +682,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_gbtrf_wide(Geo g, double *__res
 
 // Returns BANDLU_OK after a launch, BANDLU_NOT_BANDED when the kernel cannot be
 // made resident (the caller then takes another kernel), or BANDLU_ERR_CUDA.
-template <int RPT>
+template <int CW, int RPT>
 int launch_rpt(const Geo &g, int grid, size_t smem, double *AB, int *ipiv, int *d_info, int *flags, cudaStream_t s) {
+  constexpr int kThreads = Lay<CW>::kThreads;
   static bool attr = false;
   if (!attr) {
-    if (cudaFuncSetAttribute(k_gbtrf_wide<RPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
+    if (cudaFuncSetAttribute(k_gbtrf_wide<CW, RPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
         cudaSuccess)
       return BANDLU_ERR_CUDA;
     attr = true;
   }
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_gbtrf_wide<RPT>, kThreads, smem) != cudaSuccess)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_gbtrf_wide<CW, RPT>, kThreads, smem) != cudaSuccess)
     return BANDLU_ERR_CUDA;
   if (per_sm < 1) return BANDLU_NOT_BANDED;
   Geo gg = g;
   void *args[] = {&gg, &AB, &ipiv, &d_info, &flags};
-  if (cudaLaunchCooperativeKernel((const void *)k_gbtrf_wide<RPT>, dim3(grid), dim3(kThreads), args, smem, s) !=
+  if (cudaLaunchCooperativeKernel((const void *)k_gbtrf_wide<CW, RPT>, dim3(grid), dim3(kThreads), args, smem, s) !=
       cudaSuccess)
     return BANDLU_ERR_CUDA;
   return BANDLU_OK;
@@ -690,7 +706,7 @@ int launch_rpt(const Geo &g, int grid, size_t smem, double *AB, int *ipiv, int *
 
 }  // namespace
 
-// Launch conditions: kv >= 2*kNB, at most 4 panel rows per compute thread,
+// Launch conditions: kv >= 2*kNB, at most 4 panel rows per compute thread (of 9 warps),
 // shared memory for three blocks and two panels of multipliers, and an update
 // CTA never holding more than kMaxActive blocks.  *used = false when the shape
 // does not qualify (the caller then takes another kernel).
@@ -699,7 +715,11 @@ int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *
   *used = false;
   const long long kv = (long long)kl + ku;
   if (n < 4 * kNB || n > INT_MAX / 2 || kl < 1 || kv < 2 * kNB || ldab > INT_MAX / kNB) return BANDLU_OK;
-  const int rpt = (kl + kNB + kCT - 1) / kCT;
+  // compute group: the fewest warps (2, 4 or 9) giving every panel row a thread,
+  // else 9 warps with 2 or 4 rows per thread
+  const int rows = kl + kNB;
+  const int cw = rows <= 64 ? 2 : (rows <= 128 ? 4 : 9);
+  const int rpt = (rows + 32 * cw - 1) / (32 * cw);
   if (rpt > 4) return BANDLU_OK;
   const size_t smem = ((size_t)kPanelBufs * kNB * (size_t)ldab + 2 * (size_t)kNB * kl) * sizeof(double);
   if (smem > 200 * 1024) return BANDLU_OK;
@@ -728,12 +748,16 @@ int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *
     return BANDLU_ERR_CUDA;
   }
   int rc;
-  if (rpt == 1)
-    rc = launch_rpt<1>(g, sms, smem, AB, ipiv, d_info, flags, s);
+  if (cw == 2)
+    rc = launch_rpt<2, 1>(g, sms, smem, AB, ipiv, d_info, flags, s);
+  else if (cw == 4)
+    rc = launch_rpt<4, 1>(g, sms, smem, AB, ipiv, d_info, flags, s);
+  else if (rpt == 1)
+    rc = launch_rpt<9, 1>(g, sms, smem, AB, ipiv, d_info, flags, s);
   else if (rpt == 2)
-    rc = launch_rpt<2>(g, sms, smem, AB, ipiv, d_info, flags, s);
+    rc = launch_rpt<9, 2>(g, sms, smem, AB, ipiv, d_info, flags, s);
   else
-    rc = launch_rpt<4>(g, sms, smem, AB, ipiv, d_info, flags, s);
+    rc = launch_rpt<9, 4>(g, sms, smem, AB, ipiv, d_info, flags, s);
   if (cudaFreeAsync(flags, s) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
   if (rc == BANDLU_NOT_BANDED) return BANDLU_OK;
   if (rc != BANDLU_OK) return rc;
