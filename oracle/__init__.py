@@ -64,6 +64,7 @@ def _load():
         lib.oracle_band_residual.argtypes = [i64, i32, i32, dp, i64, dp, i64, ip, dp, dp]
         lib.oracle_band_residual.restype = ctypes.c_double
         lib.oracle_is_banded.argtypes = [i64, i32, i32, i64]
+        lib.oracle_gbtrs.argtypes = [i64, i32, i32, i64, dp, i64, ip, dp, i64]
         lib.oracle_dispatch_lu_batched.argtypes = [dp, i64, i64, i64, i64, dp, i64, i64, ip, i64, ip, ip, ip, ip]
         lib.oracle_dispatch_lu_batched.restype = None
         _lib = lib
@@ -133,6 +134,22 @@ def gbtrf(AB: np.ndarray, kl: int, ku: int) -> tuple[np.ndarray, np.ndarray, int
     if info < 0:
         raise ValueError("oracle_gbtrf: bad argument")
     return AB, ipiv, info, fl.value
+
+
+def gbtrs(ABf: np.ndarray, ipiv: np.ndarray, kl: int, ku: int, B: np.ndarray) -> np.ndarray:
+    """Solve A X = B with the factors of gbtrf; B (and the result) has shape (nrhs, ldb), row c
+    being right-hand side c (column-major ldb x nrhs storage).  Returns X."""
+    ABf = np.ascontiguousarray(ABf, dtype=np.float64)
+    ipiv = np.ascontiguousarray(ipiv, dtype=np.int32)
+    X = np.array(B, dtype=np.float64, order="C", copy=True)
+    if X.ndim == 1:
+        X = X[None]
+    n, ldab = ABf.shape
+    nrhs, ldb = X.shape
+    rc = _load().oracle_gbtrs(n, kl, ku, nrhs, _dptr(ABf), ldab, _iptr(ipiv), _dptr(X), max(ldb, 1))
+    if rc != 0:
+        raise ValueError("oracle_gbtrs: bad argument")
+    return X
 
 
 def getrf_dense(A: np.ndarray) -> tuple[np.ndarray, np.ndarray, int]:

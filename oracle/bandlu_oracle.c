@@ -26,6 +26,7 @@
  *   oracle_getrf_dense        pinned (LAPACK dgetrf; exact rational elimination)
  *   oracle_band_residual      pinned (dense reconstruction with a library matmul)
  *   oracle_is_banded          pinned (the worked cases of the speedup constraint, Eq. su-con)
+ *   oracle_gbtrs              pinned (LAPACK dgbtrs; dense solve; exact rational solution; closed form)
  */
 #include <math.h>
 #include <stdint.h>
@@ -299,6 +300,56 @@ int oracle_is_banded(int64_t n, int kl, int ku, int64_t ldab)
     __int128 f = N * L * (2 * (L + U) + 1);
     __int128 F3 = 2 * N * N * N; /* 3*F */
     return 3 * (I + C + f) < F3 ? 1 : 0;
+}
+
+/*
+ * The solve after the factorisation: the backslash operator that the dispatch of
+ * Listing 1 stands for (Sec. I-A; LAPACK xGBTRS, no transpose).  Solves A X = B
+ * with A = P0 L0 P1 L1 ... U as left by oracle_gbtrf.  B is COLUMN-major
+ * n x nrhs, leading dimension ldb >= n, and is overwritten with X.
+ *   forward, j = 0..n-2 (kl > 0): interchange rows j and ipiv[j]-1 of B; then,
+ *     for each right-hand side with b = B(j) != 0,
+ *     B(j+t) = fma(-l_{j+t,j}, b, B(j+t)) for t = 1..min(kl, n-1-j), the
+ *     multipliers being AB(kv+t, j);
+ *   backward, j = n-1..0: if B(j) != 0: B(j) = B(j) / U(j,j), then
+ *     B(i) = fma(-B(j), U(i,j), B(i)) for i = max(0, j-kv)..j-1, U(i,j) = AB(kv+i-j, j).
+ * The zero tests are those of the reference BLAS (xGER skips a zero element of
+ * its y vector, xTBSV a zero element of x).  Returns 0, or -1 on a bad argument.
+ */
+int oracle_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab,
+                 const int *ipiv, double *B, int64_t ldb)
+{
+    if (n < 0 || kl < 0 || ku < 0 || nrhs < 0 || ldab < 2 * (int64_t)kl + ku + 1 || ldb < (n > 1 ? n : 1))
+        return -1;
+    const int64_t kv = (int64_t)kl + ku;
+#define AB_(r, c) AB[(r) + (c) * ldab]
+    for (int64_t c = 0; c < nrhs; ++c) {
+        double *b = B + c * ldb;
+        if (kl > 0) {
+            for (int64_t j = 0; j + 1 < n; ++j) {
+                const int64_t km = (int64_t)kl < n - 1 - j ? (int64_t)kl : n - 1 - j;
+                const int64_t l = ipiv[j] - 1;
+                if (l != j) {
+                    const double t0 = b[l];
+                    b[l] = b[j];
+                    b[j] = t0;
+                }
+                const double bj = b[j];
+                if (bj != 0.0)
+                    for (int64_t t = 1; t <= km; ++t) b[j + t] = fma(-AB_(kv + t, j), bj, b[j + t]);
+            }
+        }
+        for (int64_t j = n - 1; j >= 0; --j) {
+            if (b[j] != 0.0) {
+                b[j] = b[j] / AB_(kv, j);
+                const double x = b[j];
+                const int64_t i0 = j - kv > 0 ? j - kv : 0;
+                for (int64_t i = i0; i < j; ++i) b[i] = fma(-x, AB_(kv + i - j, j), b[i]);
+            }
+        }
+    }
+#undef AB_
+    return 0;
 }
 
 /*

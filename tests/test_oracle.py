@@ -159,6 +159,90 @@ def test_gbtrf_matches_lapack_dgbtrf(oracle_mod):
             assert np.max(np.abs(ABf - ref)) / scale < 1e-13, (n, kl, ku, dist)
 
 
+# ----------------------------------------------------------------------------------------------
+# The solve after the factorisation (the backslash of Listing 1; LAPACK xGBTRS)
+# ----------------------------------------------------------------------------------------------
+
+def test_gbtrs_matches_lapack_dgbtrs(oracle_mod):
+    """LAPACK's dgbtrs on the same factors and right-hand sides: the same solution to rounding."""
+    cases = [(1, 0, 0), (2, 1, 0), (8, 1, 1), (37, 3, 2), (64, 16, 16), (200, 8, 30), (128, 0, 4),
+             (128, 5, 0), (96, 31, 31)]
+    for idx, (n, kl, ku) in enumerate(cases):
+        A = rand_banded(n, kl, ku, seed=300 + idx, dist="normal", boost=2.0)
+        ABf, ipiv, info, _ = oracle_mod.gbtrf(oracle_mod.dense_to_band(A, kl, ku), kl, ku)
+        assert info == 0
+        B = np.random.default_rng(idx).standard_normal((3, n))
+        X = oracle_mod.gbtrs(ABf, ipiv, kl, ku, B)
+        xl, linfo = lapack.dgbtrs(lapack_layout(ABf), kl, ku, B.T.copy(), ipiv - 1)
+        assert linfo == 0
+        assert np.max(np.abs(X - xl.T)) <= 1e-12 * max(np.max(np.abs(xl)), 1.0), (n, kl, ku)
+
+
+def test_gbtrs_backward_error(oracle_mod):
+    """||A X - B|| / (||A|| ||X|| n eps) stays small, against a library dense product."""
+    for idx, (n, kl, ku) in enumerate([(300, 4, 6), (500, 16, 16), (400, 40, 3)]):
+        A = rand_banded(n, kl, ku, seed=400 + idx, dist="uniform")
+        ABf, ipiv, info, _ = oracle_mod.gbtrf(oracle_mod.dense_to_band(A, kl, ku), kl, ku)
+        B = np.random.default_rng(idx).uniform(-1, 1, (2, n))
+        X = oracle_mod.gbtrs(ABf, ipiv, kl, ku, B)
+        for c in range(2):
+            r = np.max(np.abs(A @ X[c] - B[c]))
+            bound = np.max(np.sum(np.abs(A), axis=1)) * np.max(np.abs(X[c])) * n * 2.0 ** -53
+            assert r / bound <= 10.0, (n, kl, ku, r / bound)
+
+
+def test_gbtrs_exact_rational_solutions(oracle_mod):
+    """Small integer systems solved exactly in rationals: the oracle's solution to rounding."""
+    from fractions import Fraction
+    rng = np.random.default_rng(5)
+    for trial in range(40):
+        n, kl, ku = int(rng.integers(1, 9)), int(rng.integers(0, 3)), int(rng.integers(0, 3))
+        A = np.zeros((n, n))
+        for i in range(n):
+            for j in range(max(0, i - kl), min(n, i + ku + 1)):
+                A[i, j] = float(rng.integers(-4, 5))
+            A[i, i] = float(rng.integers(5, 9)) * (1 if rng.random() < 0.5 else -1)
+        b = rng.integers(-9, 10, n).astype(float)
+        # exact elimination with rationals
+        M = [[Fraction(int(A[i, j])) for j in range(n)] + [Fraction(int(b[i]))] for i in range(n)]
+        for j in range(n):
+            p = max(range(j, n), key=lambda r: abs(M[r][j]))
+            M[j], M[p] = M[p], M[j]
+            for r in range(j + 1, n):
+                f = M[r][j] / M[j][j]
+                M[r] = [x - f * y for x, y in zip(M[r], M[j])]
+        x = [Fraction(0)] * n
+        for j in reversed(range(n)):
+            x[j] = (M[j][n] - sum(M[j][k] * x[k] for k in range(j + 1, n))) / M[j][j]
+        ABf, ipiv, info, _ = oracle_mod.gbtrf(oracle_mod.dense_to_band(A, kl, ku), kl, ku)
+        X = oracle_mod.gbtrs(ABf, ipiv, kl, ku, b[None])[0]
+        ex = np.array([float(v) for v in x])
+        assert np.max(np.abs(X - ex)) <= 1e-13 * max(np.max(np.abs(ex)), 1.0), (trial, n, kl, ku)
+
+
+@pytest.mark.parametrize("n", [1, 2, 10, 100])
+def test_gbtrs_tridiagonal_closed_form(oracle_mod, n):
+    """tridiag(-1, 2, -1) x = e_1 has x_i = (n - i) / (n + 1) (0-based i)."""
+    A = np.diag(np.full(n, 2.0)) - np.diag(np.ones(n - 1), 1) - np.diag(np.ones(n - 1), -1)
+    ABf, ipiv, info, _ = oracle_mod.gbtrf(oracle_mod.dense_to_band(A, 1, 1), 1, 1)
+    e1 = np.zeros(n); e1[0] = 1.0
+    X = oracle_mod.gbtrs(ABf, ipiv, 1, 1, e1[None])[0]
+    ex = (n - np.arange(n)) / (n + 1.0)
+    assert np.max(np.abs(X - ex)) <= 4 * n * 2.0 ** -52
+
+
+def test_gbtrs_zero_right_hand_side_and_layout(oracle_mod):
+    n, kl, ku = 60, 3, 2
+    A = rand_banded(n, kl, ku, seed=9, boost=1.0)
+    ABf, ipiv, info, _ = oracle_mod.gbtrf(oracle_mod.dense_to_band(A, kl, ku), kl, ku)
+    Z = oracle_mod.gbtrs(ABf, ipiv, kl, ku, np.zeros((2, n)))
+    assert np.all(Z == 0.0) and not np.any(np.signbit(Z))   # every step skipped: +0.0 stays +0.0
+    B = np.random.default_rng(1).standard_normal((2, n + 5))  # ldb = n + 5: the padding is untouched
+    X = oracle_mod.gbtrs(ABf, ipiv, kl, ku, B)
+    assert np.array_equal(X[:, n:], B[:, n:])
+    assert np.allclose(A @ X[0, :n], B[0, :n], atol=1e-12)
+
+
 def factors_from_band(ABf, kl, ku):
     """U (dense, upper) and the multiplier matrix (dense, strictly lower) from band storage."""
     n = ABf.shape[0]

@@ -39,6 +39,11 @@ MUTANTS = [
     ("flops_drop_reciprocal", "fl += 1 + km + 2 * km * (ju - j);", "fl += km + 2 * km * (ju - j);"),
     ("dense_lu_swaps_whole_row", "for (int64_t c = j; c < n; ++c) {\n                    double t0 = A[j * lda + c];",
      "for (int64_t c = 0; c < n; ++c) {\n                    double t0 = A[j * lda + c];"),
+    ("gbtrs_no_interchange", "if (l != j) {\n                    const double t0 = b[l];",
+     "if (0) {\n                    const double t0 = b[l];"),
+    ("gbtrs_update_sign", "b[j + t] = fma(-AB_(kv + t, j), bj, b[j + t]);", "b[j + t] = fma(AB_(kv + t, j), bj, b[j + t]);"),
+    ("gbtrs_drops_last_multiplier", "for (int64_t t = 1; t <= km; ++t) b[j + t]", "for (int64_t t = 1; t < km; ++t) b[j + t]"),
+    ("gbtrs_drops_top_superdiagonal", "const int64_t i0 = j - kv > 0 ? j - kv : 0;", "const int64_t i0 = j - kv + 1 > 0 ? j - kv + 1 : 0;"),
 ]
 
 
