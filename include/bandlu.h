@@ -121,6 +121,41 @@ int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t lda
                 int *h_ku, int *d_info, cudaStream_t stream);
 
 /*
+ * gbtrs -- the solve after the factorisation: the backslash operator the
+ * dispatch of Listing 1 (Sec. I-A) stands for, on the band path (LAPACK xGBTRS,
+ * no transpose).  Solves A X = B with A = P0 L0 P1 L1 ... U as left in AB and
+ * ipiv by gbtrf (same kl, ku, ldab).
+ *   forward, j = 0..n-2 (kl > 0): rows j and ipiv[j]-1 of B are interchanged;
+ *     then, where b = B(j, c) != 0, B(j+t, c) = fma(-l_{j+t,j}, b, B(j+t, c)) for
+ *     t = 1..min(kl, n-1-j);
+ *   backward, j = n-1..0: where B(j, c) != 0, B(j, c) = B(j, c) / U(j,j) and
+ *     B(i, c) = fma(-B(j, c), U(i,j), B(i, c)) for i = max(0, j-kl-ku)..j-1.
+ * (The zero tests are those of the reference BLAS.)  A singular U (a zero
+ * U(j,j)) yields infinities or NaNs, as in LAPACK; callers check info first.
+ * Arguments (all DEVICE pointers): 1 n >= 0, 2 kl >= 0, 3 ku >= 0, 4 nrhs >= 0,
+ * 5 AB (read only), 6 ldab >= 2*kl+ku+1, 7 ipiv (1-based, read only),
+ * 8 B (COLUMN-major n x nrhs, overwritten with X), 9 ldb >= max(1, n).
+ * Returns BANDLU_OK, -i for a bad argument i, BANDLU_ERR_CUDA.  Asynchronous.
+ */
+int gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
+          int64_t ldb, cudaStream_t stream);
+
+/*
+ * dispatch_solve -- A X = B through the structure-aware dispatch: dispatch_lu,
+ * then, on the band path, gbtrs with the factors it produced (the backslash of
+ * Listing 1 with the dense branch left to the caller).
+ * Returns what dispatch_lu returns.  On BANDLU_OK the solve is enqueued on
+ * `stream`; it reads *d_info on the device and leaves B as it is when the
+ * factor is singular (info > 0), so no further host synchronisation is needed.
+ * On BANDLU_NOT_BANDED nothing further is enqueued and B is untouched.
+ * Arguments: 1 A, 2 n, 3 lda, 4 B (COLUMN-major n x nrhs), 5 ldb >= max(1, n),
+ * 6 nrhs >= 0, 7 AB, 8 ldab >= 1, 9 ipiv, 10 h_kl, 11 h_ku (HOST), 12 d_info.
+ * Scratch: as dispatch_lu.
+ */
+int dispatch_solve(const double *A, int64_t n, int64_t lda, double *B, int64_t ldb, int64_t nrhs, double *AB,
+                   int64_t ldab, int *ipiv, int *h_kl, int *h_ku, int *d_info, cudaStream_t stream);
+
+/*
  * dispatch_lu_batched -- the strategy of Sec. II-A applied to `batch`
  * independent n x n matrices in one call, with no host round trip.
  *

@@ -57,7 +57,10 @@ def load():
         lib.dispatch_lu.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
         lib.dispatch_lu_noalloc.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
         lib.dispatch_lu_batched.argtypes = [vp, i64, i64, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
-        for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "dispatch_lu", "dispatch_lu_batched",
+        lib.gbtrs.argtypes = [i64, i32, i32, i64, vp, i64, vp, vp, i64, vp]
+        lib.dispatch_solve.argtypes = [vp, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
+        for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "gbtrs", "dispatch_lu", "dispatch_solve",
+                  "dispatch_lu_batched",
                   "dispatch_lu_noalloc"):
             getattr(lib, f).restype = ctypes.c_int
         lib.bandlu_selftest_rcp_host.argtypes = [vp, vp, i64]
@@ -108,6 +111,19 @@ def dispatch_lu(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -
     kl, ku = ctypes.c_int(-1), ctypes.c_int(-1)
     rc = load().dispatch_lu(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), ctypes.addressof(kl),
                             ctypes.addressof(ku), _ptr(d_info), _stream(stream))
+    return rc, kl.value, ku.value
+
+
+def gbtrs(n: int, kl: int, ku: int, nrhs: int, AB, ldab: int, ipiv, B, ldb: int, stream=None) -> int:
+    return load().gbtrs(n, kl, ku, nrhs, _ptr(AB), ldab, _ptr(ipiv), _ptr(B), ldb, _stream(stream))
+
+
+def dispatch_solve(A, n: int, lda: int, B, ldb: int, nrhs: int, AB, ldab: int, ipiv, d_info,
+                   stream=None) -> tuple[int, int, int]:
+    """Returns (status, kl, ku); kl and ku are the host outputs of the C call."""
+    kl, ku = ctypes.c_int(-1), ctypes.c_int(-1)
+    rc = load().dispatch_solve(_ptr(A), n, lda, _ptr(B), ldb, nrhs, _ptr(AB), ldab, _ptr(ipiv),
+                               ctypes.addressof(kl), ctypes.addressof(ku), _ptr(d_info), _stream(stream))
     return rc, kl.value, ku.value
 
 

@@ -1,5 +1,5 @@
 // api.cu -- the C ABI (declared in include/bandlu.h): argument checks, then the
-// launches of detect.cu, convert.cu, gbtrf.cu and batched.cu.
+// launches of detect.cu, convert.cu, gbtrf.cu, gbtrf_wide.cu, gbtrs.cu and batched.cu.
 #include <climits>
 
 #include "common.cuh"
@@ -74,6 +74,42 @@ int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t lda
   rc = bandlu::launch_dense_to_band(A, lda, n, h[0], h[1], AB, ldab, stream);
   if (rc != BANDLU_OK) return rc;
   return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream);
+}
+
+int gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
+          int64_t ldb, cudaStream_t stream) {
+  const bool work = n > 0 && nrhs > 0;
+  if (bad_n(n)) return -1;
+  if (kl < 0) return -2;
+  if (ku < 0) return -3;
+  if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -4;
+  if (AB == nullptr && work) return -5;
+  if (ldab < 2 * (int64_t)kl + ku + 1) return -6;
+  if (ipiv == nullptr && work) return -7;
+  if (B == nullptr && work) return -8;
+  if (ldb < max1(n)) return -9;
+  return bandlu::launch_gbtrs(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, nullptr, stream);
+}
+
+int dispatch_solve(const double *A, int64_t n, int64_t lda, double *B, int64_t ldb, int64_t nrhs, double *AB,
+                   int64_t ldab, int *ipiv, int *h_kl, int *h_ku, int *d_info, cudaStream_t stream) {
+  const bool work = n > 0 && nrhs > 0;
+  if (A == nullptr && n > 0) return -1;
+  if (bad_n(n)) return -2;
+  if (lda < max1(n)) return -3;
+  if (B == nullptr && work) return -4;
+  if (ldb < max1(n)) return -5;
+  if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -6;
+  if (AB == nullptr && n > 0) return -7;
+  if (ldab < 1) return -8;
+  if (ipiv == nullptr && n > 0) return -9;
+  if (h_kl == nullptr) return -10;
+  if (h_ku == nullptr) return -11;
+  if (d_info == nullptr) return -12;
+  const int rc = dispatch_lu(A, n, lda, AB, ldab, ipiv, h_kl, h_ku, d_info, stream);
+  if (rc != BANDLU_OK) return rc;  // BANDLU_NOT_BANDED: B untouched, the caller solves densely
+  // the solve reads info on the device and leaves B as it is for a singular factor
+  return bandlu::launch_gbtrs(n, *h_kl, *h_ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, stream);
 }
 
 int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,

@@ -104,6 +104,9 @@ int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv,
                  bool allow_alloc = true);
 int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s,
                       bool *used);
+// d_info: when not null and *d_info != 0 (a singular factor), B is left as it is.
+int launch_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
+                 int64_t ldb, const int *d_info, cudaStream_t s);
 int launch_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,
                    int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku, int *d_info,
                    int *d_status, cudaStream_t s);

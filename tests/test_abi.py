@@ -31,7 +31,8 @@ def test_library_builds_and_exports_every_declared_symbol():
     assert os.path.exists(path)
     lib = ctypes.CDLL(path)
     names = declared_functions()
-    assert {"detect_bandwidth", "dense_to_band", "gbtrf", "dispatch_lu", "dispatch_lu_batched"} <= set(names)
+    assert {"detect_bandwidth", "dense_to_band", "gbtrf", "gbtrs", "dispatch_lu", "dispatch_solve",
+            "dispatch_lu_batched"} <= set(names)
     for name in names:
         assert hasattr(lib, name), name
     assert bandlu.version().startswith("bandlu")
@@ -102,6 +103,38 @@ def test_dispatch_lu_argument_checks(args, expect):
 ])
 def test_dispatch_lu_batched_argument_checks(args, expect):
     assert bandlu.dispatch_lu_batched(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((-1, 1, 1, 1, DEV, 4, DEV, DEV, 4), -1),
+    ((4, -1, 1, 1, DEV, 4, DEV, DEV, 4), -2),
+    ((4, 1, -1, 1, DEV, 4, DEV, DEV, 4), -3),
+    ((4, 1, 1, -1, DEV, 4, DEV, DEV, 4), -4),
+    ((4, 1, 1, 1, 0, 4, DEV, DEV, 4), -5),
+    ((4, 2, 1, 1, DEV, 5, DEV, DEV, 4), -6),
+    ((4, 1, 1, 1, DEV, 4, 0, DEV, 4), -7),
+    ((4, 1, 1, 1, DEV, 4, DEV, 0, 4), -8),
+    ((4, 1, 1, 1, DEV, 4, DEV, DEV, 3), -9),
+])
+def test_gbtrs_argument_checks(args, expect):
+    assert bandlu.gbtrs(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, DEV, 4, 1, DEV, 4, DEV, DEV), -1),
+    ((DEV, -2, 4, DEV, 4, 1, DEV, 4, DEV, DEV), -2),
+    ((DEV, 4, 3, DEV, 4, 1, DEV, 4, DEV, DEV), -3),
+    ((DEV, 4, 4, 0, 4, 1, DEV, 4, DEV, DEV), -4),
+    ((DEV, 4, 4, DEV, 3, 1, DEV, 4, DEV, DEV), -5),
+    ((DEV, 4, 4, DEV, 4, -1, DEV, 4, DEV, DEV), -6),
+    ((DEV, 4, 4, DEV, 4, 1, 0, 4, DEV, DEV), -7),
+    ((DEV, 4, 4, DEV, 4, 1, DEV, 0, DEV, DEV), -8),
+    ((DEV, 4, 4, DEV, 4, 1, DEV, 4, 0, DEV), -9),
+    ((DEV, 4, 4, DEV, 4, 1, DEV, 4, DEV, 0), -12),
+])
+def test_dispatch_solve_argument_checks(args, expect):
+    rc, _, _ = bandlu.dispatch_solve(*args, stream=0)
+    assert rc == expect
 
 
 def test_binding_has_the_c_names():

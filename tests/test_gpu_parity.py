@@ -308,6 +308,98 @@ def test_batched_nan_candidates(n, kl, ku):
 
 
 # --------------------------------------------------------------------------------------------
+# gbtrs (the solve after the factorisation) and dispatch_solve
+# --------------------------------------------------------------------------------------------
+
+def gbtrs_gpu(ABf, ipiv, kl, ku, B):
+    n, ldab = ABf.shape
+    nrhs, ldb = B.shape
+    ABd = torch.from_numpy(np.ascontiguousarray(ABf)).to(DEV)
+    ipd = torch.from_numpy(np.ascontiguousarray(ipiv, dtype=np.int32)).to(DEV)
+    Bd = torch.from_numpy(np.ascontiguousarray(B)).to(DEV)
+    rc = bandlu.gbtrs(n, kl, ku, nrhs, ABd, ldab, ipd, Bd, ldb)
+    torch.cuda.synchronize()
+    assert rc == 0, rc
+    return Bd.cpu().numpy()
+
+
+def assert_same_solution(got, ref):
+    nan_g, nan_r = np.isnan(got), np.isnan(ref)
+    assert np.array_equal(nan_g, nan_r)
+    if not np.array_equal(got[~nan_g].view(np.int64), ref[~nan_r].view(np.int64)):
+        d = np.argwhere(got.view(np.int64) != ref.view(np.int64))[0]
+        raise AssertionError(f"solution not bit-identical first at {tuple(d)}: {got[tuple(d)]!r} vs {ref[tuple(d)]!r}")
+
+
+# windows of 1, 2, 4, 8 and 16 registers per lane, and the generic path (kl+ku+1 > 512)
+@pytest.mark.parametrize("n,kl,ku,nrhs", [(1, 0, 0, 1), (2, 1, 0, 1), (17, 3, 5, 3), (300, 2, 2, 1), (512, 3, 3, 2),
+                                          (1000, 16, 16, 5), (700, 0, 12, 1), (700, 12, 0, 1), (600, 40, 40, 2),
+                                          (500, 60, 60, 1), (400, 100, 150, 1), (350, 200, 250, 1),
+                                          (250, 300, 300, 1)])
+def test_gbtrs_matches_oracle(n, kl, ku, nrhs):
+    A = banded(n, kl, ku, seed=3 * n + kl + ku, dist="normal").numpy()
+    ABf, ipiv, info, _ = oracle.gbtrf(oracle.dense_to_band(A, kl, ku), kl, ku)
+    B = np.random.default_rng(n + nrhs).standard_normal((nrhs, n + 3))   # ldb = n + 3
+    B[:, :2] = 0.0                                                       # the zero skips
+    ref = oracle.gbtrs(ABf, ipiv, kl, ku, B)
+    assert_same_solution(gbtrs_gpu(ABf, ipiv, kl, ku, B), ref)
+
+
+def test_gbtrs_zero_right_hand_sides_and_singular_factor():
+    n, kl, ku = 400, 5, 4
+    A = banded(n, kl, ku, seed=77).numpy()
+    ABf, ipiv, info, _ = oracle.gbtrf(oracle.dense_to_band(A, kl, ku), kl, ku)
+    B = np.zeros((3, n))
+    B[1, 7] = 1.0
+    assert_same_solution(gbtrs_gpu(ABf, ipiv, kl, ku, B), oracle.gbtrs(ABf, ipiv, kl, ku, B))
+    A[:, 100] = 0.0                                                      # singular: infinities, NaNs
+    ABf, ipiv, info, _ = oracle.gbtrf(oracle.dense_to_band(A, kl, ku), kl, ku)
+    assert info > 0
+    B = np.random.default_rng(2).standard_normal((1, n))
+    assert_same_solution(gbtrs_gpu(ABf, ipiv, kl, ku, B), oracle.gbtrs(ABf, ipiv, kl, ku, B))
+
+
+def run_solve(A, B, ldab):
+    n, lda = A.shape
+    nrhs, ldb = B.shape
+    Ad, Bd = A.to(DEV), torch.from_numpy(np.ascontiguousarray(B)).to(DEV)
+    AB = torch.zeros((n, ldab), dtype=torch.float64, device=DEV)
+    ipiv = torch.zeros(max(n, 1), dtype=torch.int32, device=DEV)
+    info = torch.full((1,), -5, dtype=torch.int32, device=DEV)
+    rc, kl, ku = bandlu.dispatch_solve(Ad, n, lda, Bd, ldb, nrhs, AB, ldab, ipiv, info)
+    torch.cuda.synchronize()
+    return rc, kl, ku, Bd.cpu().numpy(), int(info.item())
+
+
+@pytest.mark.parametrize("n,kl,ku", [(512, 3, 3), (4096, 16, 16), (1500, 40, 20)])
+def test_dispatch_solve_matches_oracle(n, kl, ku):
+    A = banded(n, kl, ku, seed=n + 1)
+    ldab = 2 * kl + ku + 1
+    B = np.random.default_rng(n).uniform(-1, 1, (2, n))
+    rc, gkl, gku, X, info = run_solve(A, B, ldab)
+    r = oracle.dispatch_lu(A.numpy(), ldab)
+    assert (rc, gkl, gku, info) == (r["status"], r["kl"], r["ku"], r["info"]) == (0, kl, ku, 0)
+    ref = oracle.gbtrs(r["AB"], r["ipiv"], kl, ku, B)
+    assert_same_solution(X, ref)
+    An = A.numpy()
+    r = np.max(np.abs(An @ X[0] - B[0]))
+    assert r / (np.max(np.sum(np.abs(An), axis=1)) * np.max(np.abs(X[0])) * n * 2.0 ** -53) <= 10.0
+
+
+def test_dispatch_solve_declines_and_skips_singular():
+    n = 300
+    A = banded(n, 2, 3, seed=4)
+    A[n - 1, 0] = 1e-3                                                   # not banded: B untouched
+    B = np.random.default_rng(0).standard_normal((1, n))
+    rc, kl, ku, X, info = run_solve(A, B, 8)
+    assert rc == bandlu.BANDLU_NOT_BANDED and np.array_equal(X, B) and info == -5
+    A = banded(n, 2, 3, seed=4)
+    A[:, 50] = 0.0                                                       # singular: B untouched, info > 0
+    rc, kl, ku, X, info = run_solve(A, B, 8)
+    assert rc == 0 and info == 51 and np.array_equal(X, B)
+
+
+# --------------------------------------------------------------------------------------------
 # dispatch_lu and dispatch_lu_batched
 # --------------------------------------------------------------------------------------------
 
