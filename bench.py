@@ -507,9 +507,18 @@ def run_workload_report(args):
             t_conv = timed(conv, reps)
             t_fac = timed(fac, max(1, min(reps, 5))) if n > 20000 else timed(fac, reps)
             flops = band_flops(ipiv.cpu().numpy(), AB2[:, kl + ku].cpu().numpy(), n, kl, ku)
+            # the solve with the factors, one right-hand side (forward and back substitution)
+            xb = torch.empty(n, dtype=torch.float64, device=dev)
+            b0 = torch.linspace(-1.0, 1.0, n, dtype=torch.float64, device=dev)
+
+            def sol():
+                xb.copy_(b0)
+                bandlu.check(bandlu.gbtrs(n, kl, ku, 1, AB2, ldab, ipiv, xb, n, stream), "gbtrs")
+            t_sol = timed(sol, max(1, min(reps, 5)))
             out.update({"convert_us": t_conv * 1e6, "gbtrf_ms": t_fac * 1e3, "gbtrf_gflops": flops / t_fac / 1e9,
                         "gbtrf_ns_per_column": t_fac / n * 1e9, "flops": flops,
-                        "gflops_dispatch": flops / t_disp / 1e9})
+                        "gflops_dispatch": flops / t_disp / 1e9, "gbtrs_1rhs_ms": t_sol * 1e3,
+                        "gbtrs_ns_per_row": t_sol / n * 1e9})
         if n <= 20000:
             d_ms = dense_lu_ms(torch, A, stream)
             out["dense_lu_ms"] = d_ms

@@ -214,6 +214,75 @@ __global__ void __launch_bounds__(128) k_gbtrs_generic(int n, int kl, int ku, in
   }
 }
 
+// Wide bands: one CTA per right-hand side.  The active part of b lives in a
+// shared-memory ring of WS rows (a power of two >= kl+ku+1+32; row i in slot
+// i mod WS).  Forward, the ring holds rows j..j+WS-1; backward, rows
+// j-WS+1..j.  A step is one thread's interchange (or division), a barrier, the
+// threads' updates of one row each, a barrier.  Every 32 steps the 32 slots of
+// the rows just finished are refilled at once with the rows WS further on
+// (needed no earlier than ku+1 steps later, so one load latency per 32 steps).
+__global__ void __launch_bounds__(256) k_gbtrs_cta(int n, int kl, int ku, int WS, const double *__restrict__ AB,
+                                                   long long ldab, const int *__restrict__ ipiv,
+                                                   double *__restrict__ B, long long ldb,
+                                                   const int *__restrict__ d_info) {
+  extern __shared__ double ring[];  // WS
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int rhs = blockIdx.x;
+  if (d_info != nullptr && *d_info != 0) return;
+  double *b = B + (long long)rhs * ldb;
+  const long long kv = (long long)kl + ku;
+  const int mask = WS - 1;
+  if (kl > 0 && n > 1) {
+    for (int i = tid; i < WS; i += nt) ring[i] = i < n ? b[i] : 0.0;
+    __syncthreads();
+    for (int j = 0; j + 1 < n; ++j) {
+      const int km = min(kl, n - 1 - j);
+      if (j >= 32 && (j & 31) == 0 && tid < 32) {  // rows j-32..j-1 are final
+        const int r = j - 32 + tid;
+        ring[r & mask] = (r + WS < n) ? b[r + WS] : 0.0;
+      }
+      if (tid == 0) {
+        const int l = ipiv[j] - 1;
+        if (l != j) {
+          const double t0 = ring[l & mask];
+          ring[l & mask] = ring[j & mask];
+          ring[j & mask] = t0;
+        }
+      }
+      __syncthreads();
+      const double bj = ring[j & mask];
+      if (nz(bj))
+        for (int t = 1 + tid; t <= km; t += nt)
+          ring[(j + t) & mask] = fma(-AB[(kv + t) + (long long)j * ldab], bj, ring[(j + t) & mask]);
+      if (tid == 0) b[j] = bj;  // y_j
+      __syncthreads();
+    }
+    if (tid == 0) b[n - 1] = ring[(n - 1) & mask];
+    __syncthreads();
+  }
+  for (int t = tid; t < WS; t += nt) {
+    const int i = n - 1 - t;
+    if (i >= 0) ring[i & mask] = b[i];
+  }
+  __syncthreads();
+  for (int j = n - 1; j >= 0; --j) {
+    const int done = n - 1 - j;  // rows j+1..n-1 are final
+    if (done >= 32 && (done & 31) == 0 && tid < 32) {
+      const int r = j + 1 + tid;  // rows j+1..j+32
+      ring[r & mask] = (r - WS >= 0) ? b[r - WS] : 0.0;
+    }
+    double xj = ring[j & mask];
+    if (nz(xj)) {  // uniform
+      xj = xj / AB[kv + (long long)j * ldab];
+      const int lo = (int)max(0LL, (long long)j - kv);
+      for (int i = j - 1 - tid; i >= lo; i -= nt)
+        ring[i & mask] = fma(-xj, AB[(kv + i - j) + (long long)j * ldab], ring[i & mask]);
+    }
+    if (tid == 0) b[j] = xj;
+    __syncthreads();
+  }
+}
+
 template <int RW>
 int launch_rw(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
               int64_t ldb, const int *d_info, cudaStream_t s) {
@@ -237,6 +306,21 @@ int launch_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int6
     if (win <= 128) return launch_rw<4>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
     if (win <= 256) return launch_rw<8>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
     if (win <= 512) return launch_rw<16>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
+  }
+  // wider bands: a CTA per right-hand side with a shared-memory ring
+  int WS = 1;
+  while (WS < win + 32) WS <<= 1;
+  if (n <= INT_MAX / 2 && nrhs <= INT_MAX && (size_t)WS * sizeof(double) <= 96 * 1024) {
+    static bool attr = false;
+    if (!attr) {
+      if (cudaFuncSetAttribute(k_gbtrs_cta, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024) != cudaSuccess)
+        return BANDLU_ERR_CUDA;
+      attr = true;
+    }
+    k_gbtrs_cta<<<(unsigned)nrhs, 256, (size_t)WS * sizeof(double), s>>>((int)n, kl, ku, WS, AB, ldab, ipiv, B, ldb,
+                                                                        d_info);
+    BANDLU_CHECK_LAUNCH();
+    return BANDLU_OK;
   }
   const int wpb = 4;
   const long long grid = (nrhs + wpb - 1) / wpb;

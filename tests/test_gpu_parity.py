@@ -331,11 +331,12 @@ def assert_same_solution(got, ref):
         raise AssertionError(f"solution not bit-identical first at {tuple(d)}: {got[tuple(d)]!r} vs {ref[tuple(d)]!r}")
 
 
-# windows of 1, 2, 4, 8 and 16 registers per lane, and the generic path (kl+ku+1 > 512)
+# windows of 1, 2, 4, 8 and 16 registers per lane, and a CTA with a shared-memory ring (kl+ku+1 > 512,
+# n > ring: the refills)
 @pytest.mark.parametrize("n,kl,ku,nrhs", [(1, 0, 0, 1), (2, 1, 0, 1), (17, 3, 5, 3), (300, 2, 2, 1), (512, 3, 3, 2),
                                           (1000, 16, 16, 5), (700, 0, 12, 1), (700, 12, 0, 1), (600, 40, 40, 2),
                                           (500, 60, 60, 1), (400, 100, 150, 1), (350, 200, 250, 1),
-                                          (250, 300, 300, 1)])
+                                          (250, 300, 300, 1), (3000, 300, 300, 2), (2100, 7, 600, 1)])
 def test_gbtrs_matches_oracle(n, kl, ku, nrhs):
     A = banded(n, kl, ku, seed=3 * n + kl + ku, dist="normal").numpy()
     ABf, ipiv, info, _ = oracle.gbtrf(oracle.dense_to_band(A, kl, ku), kl, ku)

@@ -36,6 +36,18 @@ def test_workload_dispatch_lu(name):
     got_AB, got_ipiv = AB.cpu().numpy(), ipiv.cpu().numpy()
     assert_factor_parity(got_AB, got_ipiv, int(info.item()), ABf, ipiv_o, info_o)
     assert oracle.backward_error(An, got_AB, got_ipiv, kl, ku) <= 10.0
+    # the solve with these factors, one right-hand side, bit-identical to the oracle's
+    b = np.linspace(-1.0, 1.0, n)
+    xd = torch.from_numpy(b.copy()).to(DEV)
+    assert bandlu.gbtrs(n, kl, ku, 1, AB, ldab, ipiv, xd, n) == 0
+    torch.cuda.synchronize()
+    x_ref = oracle.gbtrs(ABf, ipiv_o, kl, ku, b[None])[0]
+    x = xd.cpu().numpy()
+    # back substitution can overflow on these random bands (n = 16384, kl = 8); infinities must
+    # match bit for bit, NaNs in position (their payloads are the platform's)
+    nan_g, nan_r = np.isnan(x), np.isnan(x_ref)
+    assert np.array_equal(nan_g, nan_r)
+    assert np.array_equal(x[~nan_g].view(np.int64), x_ref[~nan_r].view(np.int64))
 
 
 def test_workload_stray_entry_control():
