@@ -67,6 +67,10 @@ def load():
         lib.bandlu_selftest_rcp_host.restype = None
         lib.bandlu_selftest_rcp_device.argtypes = [vp, vp, i64, i32, vp]
         lib.bandlu_selftest_rcp_device.restype = ctypes.c_int
+        lib.bandlu_selftest_div_host.argtypes = [vp, vp, vp, i64]
+        lib.bandlu_selftest_div_host.restype = None
+        lib.bandlu_selftest_div_device.argtypes = [vp, vp, vp, i64, i32, vp]
+        lib.bandlu_selftest_div_device.restype = ctypes.c_int
         lib.bandlu_version.restype = ctypes.c_char_p
         lib.bandlu_version.argtypes = []
         _lib = lib
@@ -151,6 +155,16 @@ def bandlu_selftest_rcp_host(x, y, n: int) -> None:
 def bandlu_selftest_rcp_device(x, y, n: int, use_division: int, stream=None) -> int:
     """Self-test hook: the library's reciprocal (or plain division) on the device."""
     return load().bandlu_selftest_rcp_device(_ptr(x), _ptr(y), n, use_division, _stream(stream))
+
+
+def bandlu_selftest_div_host(x, d, q, n: int) -> None:
+    """Self-test hook: the library's known-divisor division on the host (host buffers of n doubles)."""
+    load().bandlu_selftest_div_host(_ptr_host(x), _ptr_host(d), _ptr_host(q), n)
+
+
+def bandlu_selftest_div_device(x, d, q, n: int, use_division: int, stream=None) -> int:
+    """Self-test hook: the library's known-divisor division (or plain division) on the device."""
+    return load().bandlu_selftest_div_device(_ptr(x), _ptr(d), _ptr(q), n, use_division, _stream(stream))
 
 
 def _ptr_host(x) -> int:

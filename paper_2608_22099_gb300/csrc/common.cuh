@@ -21,6 +21,19 @@ __device__ __forceinline__ bool nz(double x) {
   return ((((unsigned)__double2hiint(x)) << 1) | (unsigned)__double2loint(x)) != 0u;
 }
 
+// c ? a : b as one PTX select of the 64-bit patterns.  Register windows pick
+// their rows with it: a chain of plain selects on a runtime row index can be
+// turned by the compiler into an indexed array in local memory, which puts a
+// local load on every step's dependence chain.
+__device__ __forceinline__ double dsel(bool c, double a, double b) {
+  unsigned long long r;
+  asm("{\n\t.reg .pred q;\n\tsetp.ne.u32 q, %3, 0;\n\tselp.b64 %0, %1, %2, q;\n\t}"
+      : "=l"(r)
+      : "l"((unsigned long long)__double_as_longlong(a)), "l"((unsigned long long)__double_as_longlong(b)),
+        "r"((unsigned)c));
+  return __longlong_as_double((long long)r);
+}
+
 // Pivot-search key of a candidate: for non-NaN doubles |x| < |y| iff
 // key(x) < key(y).  The xGBTRF comparison order starts its running best at the
 // first candidate and replaces it only by a strictly larger modulus, which a

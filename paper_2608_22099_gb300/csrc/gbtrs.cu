@@ -7,171 +7,46 @@
 //            j+1..j+kl take fma(-l, b_j, .);
 //   backward j = n-1..0: if b_j != 0, b_j = b_j / u_jj and rows j-kv..j-1 take
 //            fma(-b_j, u, .).
-// One warp per right-hand side keeps the active part of b in registers (a
-// window of W = 32*RW rows: row t of the window on lane t % 32, register t / 32),
-// reads each step's factor column kPf steps ahead (the step loop is unrolled by
-// kPf so that every prefetch slot is one register), and writes every finished
-// entry once.  The same operations in the same order as the oracle, so the
-// solution is bit-identical to it.
+// One warp per right-hand side keeps the active part of b in registers, in a
+// window that rotates with the steps (trwin.cuh); the division by u_jj uses a
+// two-term reciprocal formed ahead of time, 32 diagonal entries at once
+// (div_known: four dependent FP64 operations instead of a full division).  The
+// same operations in the same order as the oracle, so the solution is
+// bit-identical to it.  Interchanges outside j..j+kl (not produced by gbtrf)
+// are ignored.
 #include <climits>
 
 #include "common.cuh"
+#include "rcp.cuh"
+#include "trwin.cuh"
 
 namespace bandlu {
 namespace {
 
-constexpr int kPf = 4;  // steps read ahead
-
-// Element t of the window (t warp-uniform).
-template <int RW>
-__device__ __forceinline__ double win_get(const double (&w)[RW], int t) {
-  double v = 0.0;
-#pragma unroll
-  for (int r = 0; r < RW; ++r) {
-    const double x = __shfl_sync(FULL, w[r], t & 31);
-    if (r == (t >> 5)) v = x;
-  }
-  return v;
-}
-
-template <int RW>
-__device__ __forceinline__ void win_set(double (&w)[RW], int t, double v, int lane) {
-#pragma unroll
-  for (int r = 0; r < RW; ++r)
-    if (r == (t >> 5) && lane == (t & 31)) w[r] = v;
-}
-
-// w[t] = w[t+1] for every t; the last row takes `in`.
-template <int RW>
-__device__ __forceinline__ void win_shift(double (&w)[RW], double in, int lane) {
-#pragma unroll
-  for (int r = 0; r < RW; ++r) {
-    const double carry = (r + 1 < RW) ? __shfl_sync(FULL, w[r + 1 < RW ? r + 1 : r], 0) : in;
-    const double sh = __shfl_down_sync(FULL, w[r], 1);
-    w[r] = lane == 31 ? carry : sh;
-  }
-}
-
-template <int RW>
-__global__ void __launch_bounds__(128) k_gbtrs_window(int n, int kl, int ku, int nrhs, const double *__restrict__ AB,
-                                                      int ldab, const int *__restrict__ ipiv, double *__restrict__ B,
-                                                      long long ldb, const int *__restrict__ d_info) {
-  constexpr int W = 32 * RW;
-  const int lane = threadIdx.x & 31;
+// The two sweeps of a right-hand side (trwin.cuh), one warp each, as two
+// kernels so that each gets its own window size and register allocation:
+// forward with the interchanges and the multipliers (window >= kl+1), backward
+// with U (window >= kl+ku+1).  kPf: steps read ahead.
+template <int RW, int kPf>
+__global__ void __launch_bounds__(128) k_gbtrs_fwd(int n, int kl, int ku, int nrhs, const double *__restrict__ AB,
+                                                   int ldab, const int *__restrict__ ipiv, double *__restrict__ B,
+                                                   long long ldb, const int *__restrict__ d_info) {
   const int rhs = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (rhs >= nrhs) return;  // whole warp
   if (d_info != nullptr && *d_info != 0) return;  // a singular factor: B is left as it is
-  double *b = B + (long long)rhs * ldb;
+  trwin::sweep<RW, kPf, true, true, false>(B + (long long)rhs * ldb, n, kl, trwin::GbLower{AB, ldab, kl + ku}, ipiv);
+}
+
+template <int RW, int kPf>
+__global__ void __launch_bounds__(128) k_gbtrs_bwd(int n, int kl, int ku, int nrhs, const double *__restrict__ AB,
+                                                   int ldab, double *__restrict__ B, long long ldb,
+                                                   const int *__restrict__ d_info) {
+  const int rhs = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (rhs >= nrhs) return;
+  if (d_info != nullptr && *d_info != 0) return;
   const int kv = kl + ku;
-
-  // ---------------- forward: window row t = b_{j+t} ----------------
-  if (kl > 0 && n > 1) {
-    double w[RW];
-#pragma unroll
-    for (int r = 0; r < RW; ++r) {
-      const int t = lane + 32 * r;
-      w[r] = t < n ? b[t] : 0.0;
-    }
-    // slot s: multipliers of step j = j0 + s (window row t = 1..kl) and the row
-    // entering the window after it (b_{j+W})
-    double lm[kPf][RW], en[kPf];
-    int pv[kPf];
-#pragma unroll
-    for (int s = 0; s < kPf; ++s) {
-      const int j = s;
-#pragma unroll
-      for (int r = 0; r < RW; ++r) {
-        const int t = lane + 32 * r;
-        lm[s][r] = (j < n - 1 && t >= 1 && t <= min(kl, n - 1 - j)) ? AB[(kv + t) + (long long)j * ldab] : 0.0;
-      }
-      en[s] = (lane == 31 && j + W < n) ? b[j + W] : 0.0;
-      pv[s] = j < n - 1 ? ipiv[j] - 1 - j : 0;
-    }
-    for (int j0 = 0; j0 < n - 1; j0 += kPf) {
-#pragma unroll
-      for (int s = 0; s < kPf; ++s) {
-        const int j = j0 + s;
-        if (j >= n - 1) break;
-        const int km = min(kl, n - 1 - j);
-        const int p = pv[s];
-        if (p != 0) {  // uniform
-          const double a = win_get(w, 0), c = win_get(w, p);
-          win_set(w, 0, c, lane);
-          win_set(w, p, a, lane);
-        }
-        const double bj = win_get(w, 0);
-        if (lane == 0) b[j] = bj;  // y_j
-        if (nz(bj)) {
-#pragma unroll
-          for (int r = 0; r < RW; ++r) {
-            const int t = lane + 32 * r;
-            if (t >= 1 && t <= km) w[r] = fma(-lm[s][r], bj, w[r]);
-          }
-        }
-        win_shift(w, en[s], lane);
-        // refill the slot with step j + kPf
-        const int jn = j + kPf;
-#pragma unroll
-        for (int r = 0; r < RW; ++r) {
-          const int t = lane + 32 * r;
-          lm[s][r] = (jn < n - 1 && t >= 1 && t <= min(kl, n - 1 - jn)) ? AB[(kv + t) + (long long)jn * ldab] : 0.0;
-        }
-        en[s] = (lane == 31 && jn + W < n) ? b[jn + W] : 0.0;
-        pv[s] = jn < n - 1 ? ipiv[jn] - 1 - jn : 0;
-      }
-    }
-    const double last = win_get(w, 0);
-    if (lane == 0) b[n - 1] = last;
-    __syncwarp();  // the backward sweep reads what other lanes wrote
-  }
-
-  // ---------------- backward: window row t = b_{j-t} ----------------
-  {
-    double w[RW];
-#pragma unroll
-    for (int r = 0; r < RW; ++r) {
-      const int t = lane + 32 * r;
-      w[r] = t <= n - 1 ? b[n - 1 - t] : 0.0;
-    }
-    // slot s: column j = n-1-(j0+s) of U (window row t <-> U(j-t, j) = AB(kv-t, j))
-    // and the row entering after it (b_{j-W})
-    double uc[kPf][RW], en[kPf];
-#pragma unroll
-    for (int s = 0; s < kPf; ++s) {
-      const int j = n - 1 - s;
-#pragma unroll
-      for (int r = 0; r < RW; ++r) {
-        const int t = lane + 32 * r;
-        uc[s][r] = (j >= 0 && t <= min(kv, j)) ? AB[(kv - t) + (long long)j * ldab] : 0.0;
-      }
-      en[s] = (lane == 31 && j - W >= 0) ? b[j - W] : 0.0;
-    }
-    for (int i0 = 0; i0 < n; i0 += kPf) {
-#pragma unroll
-      for (int s = 0; s < kPf; ++s) {
-        const int j = n - 1 - (i0 + s);
-        if (j < 0) break;
-        double xj = win_get(w, 0);
-        if (nz(xj)) {  // uniform
-          xj = xj / __shfl_sync(FULL, uc[s][0], 0);  // u_jj
-#pragma unroll
-          for (int r = 0; r < RW; ++r) {
-            const int t = lane + 32 * r;
-            if (t >= 1 && t <= min(kv, j)) w[r] = fma(-xj, uc[s][r], w[r]);
-          }
-        }
-        if (lane == 0) b[j] = xj;  // x_j (a zero entry stays as the updates left it)
-        win_shift(w, en[s], lane);
-        const int jn = j - kPf;
-#pragma unroll
-        for (int r = 0; r < RW; ++r) {
-          const int t = lane + 32 * r;
-          uc[s][r] = (jn >= 0 && t <= min(kv, jn)) ? AB[(kv - t) + (long long)jn * ldab] : 0.0;
-        }
-        en[s] = (lane == 31 && jn - W >= 0) ? b[jn - W] : 0.0;
-      }
-    }
-  }
+  trwin::sweep<RW, kPf, false, false, true>(B + (long long)rhs * ldb, n, kv, trwin::GbUpper{AB, ldab, kv, n},
+                                            nullptr);
 }
 
 // Any band: one warp per right-hand side, column by column through memory.
@@ -283,13 +158,47 @@ __global__ void __launch_bounds__(256) k_gbtrs_cta(int n, int kl, int ku, int WS
   }
 }
 
+// read-ahead depth for a window of 32*RW rows: kPf steps must outlast a DRAM
+// round trip (~2000 clocks)
 template <int RW>
-int launch_rw(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
-              int64_t ldb, const int *d_info, cudaStream_t s) {
+constexpr int pf_for() {
+  return RW <= 2 ? 16 : (RW <= 8 ? 8 : 4);
+}
+
+template <int RW>
+void launch_fwd(int n, int kl, int ku, int nrhs, const double *AB, int ldab, const int *ipiv, double *B, long long ldb,
+                const int *d_info, cudaStream_t s) {
   const int wpb = 4;
-  const long long grid = (nrhs + wpb - 1) / wpb;
-  k_gbtrs_window<RW><<<(unsigned)grid, 32 * wpb, 0, s>>>((int)n, kl, ku, (int)nrhs, AB, (int)ldab, ipiv, B, ldb,
-                                                         d_info);
+  k_gbtrs_fwd<RW, pf_for<RW>()><<<(unsigned)((nrhs + wpb - 1) / wpb), 32 * wpb, 0, s>>>(n, kl, ku, nrhs, AB, ldab,
+                                                                                      ipiv, B, ldb, d_info);
+}
+
+template <int RW>
+void launch_bwd(int n, int kl, int ku, int nrhs, const double *AB, int ldab, double *B, long long ldb,
+                const int *d_info, cudaStream_t s) {
+  const int wpb = 4;
+  k_gbtrs_bwd<RW, pf_for<RW>()><<<(unsigned)((nrhs + wpb - 1) / wpb), 32 * wpb, 0, s>>>(n, kl, ku, nrhs, AB, ldab,
+                                                                                      B, ldb, d_info);
+}
+
+// Register windows for both sweeps (kl+ku+1 <= 512).
+int launch_window(int n, int kl, int ku, int nrhs, const double *AB, int ldab, const int *ipiv, double *B,
+                  long long ldb, const int *d_info, cudaStream_t s) {
+  if (kl > 0 && n > 1) {
+    const int wf = kl + 1;
+    if (wf <= 32) launch_fwd<1>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
+    else if (wf <= 64) launch_fwd<2>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
+    else if (wf <= 128) launch_fwd<4>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
+    else if (wf <= 256) launch_fwd<8>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
+    else launch_fwd<16>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
+    BANDLU_CHECK_LAUNCH();
+  }
+  const int wb = kl + ku + 1;
+  if (wb <= 32) launch_bwd<1>(n, kl, ku, nrhs, AB, ldab, B, ldb, d_info, s);
+  else if (wb <= 64) launch_bwd<2>(n, kl, ku, nrhs, AB, ldab, B, ldb, d_info, s);
+  else if (wb <= 128) launch_bwd<4>(n, kl, ku, nrhs, AB, ldab, B, ldb, d_info, s);
+  else if (wb <= 256) launch_bwd<8>(n, kl, ku, nrhs, AB, ldab, B, ldb, d_info, s);
+  else launch_bwd<16>(n, kl, ku, nrhs, AB, ldab, B, ldb, d_info, s);
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;
 }
@@ -301,11 +210,7 @@ int launch_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int6
   if (n == 0 || nrhs == 0) return BANDLU_OK;
   const long long win = (long long)kl + ku + 1;  // rows the backward window needs (>= kl + 1)
   if (n <= INT_MAX / 2 && ldab <= INT_MAX && nrhs <= INT_MAX) {
-    if (win <= 32) return launch_rw<1>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
-    if (win <= 64) return launch_rw<2>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
-    if (win <= 128) return launch_rw<4>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
-    if (win <= 256) return launch_rw<8>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
-    if (win <= 512) return launch_rw<16>(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, s);
+    if (win <= 512) return launch_window((int)n, kl, ku, (int)nrhs, AB, (int)ldab, ipiv, B, ldb, d_info, s);
   }
   // wider bands: a CTA per right-hand side with a shared-memory ring
   int WS = 1;

@@ -17,6 +17,7 @@
 // ordinary division.
 #pragma once
 
+#include <cmath>
 #include <cstdint>
 #include <cstring>
 
@@ -119,6 +120,61 @@ __host__ __device__ __forceinline__ double rcp_rn(double b) {
   if (special) r = 1.0 / b;
 #endif
   return r;
+}
+
+// ---------------------------------------------------------------------------
+// x / d, correctly rounded, for a divisor known before the dividend (the
+// diagonal of U in the back substitution).  Ahead of time, off the dependence
+// chain, d gets a two-term reciprocal (div_known_prep):
+//   yh = RN(1/d)                      (rcp_rn)
+//   yl = RN(RN(1 - d*yh) * yh)        1 - d*yh is exact for a correctly rounded
+//                                     yh, so yh + yl = 1/d within ~2^-104 relative.
+// The quotient then takes four dependent floating-point operations instead of
+// a full division (Markstein's final step: P. Markstein, IBM J. Res. Dev.
+// 34(1), 1990):
+//   q0 = RN(x*yh + RN(x*yl))          within half an ulp plus 2^-50 ulp of x/d:
+//                                     a faithful quotient
+//   q  = RN(q0 + (x - d*q0)*yh)       x - d*q0 is exact for a faithful q0, and with
+//                                     yh correctly rounded this returns RN(x/d)
+// (Markstein's theorem).  No quotient of two binary64 numbers lies on a
+// rounding midpoint, so the result is the IEEE quotient bit for bit.  The
+// theorem assumes that no step overflows or underflows: div_known keeps to
+// biased exponents 64..1983 for x and d with |E(x) - E(d)| <= 900 (quotient
+// exponent within 2^-900..2^901, every remainder far above the subnormal range)
+// and takes the ordinary division otherwise (zeros, subnormals, infinities,
+// NaN, huge or tiny ratios).
+__host__ __device__ __forceinline__ int dexp(double x) { return (int)((dbits(x) >> 52) & 0x7ffull); }
+
+// Two-term reciprocal of d; *ok tells whether d is inside the range div_known
+// handles (when it is not, yh and yl are not used).
+__host__ __device__ __forceinline__ void div_known_prep(double d, double *yh, double *yl, bool *ok) {
+  const int e = dexp(d);
+  *ok = e >= 64 && e <= 1983;
+  const double h = rcp_rn(d);
+  *yh = h;
+  *yl = *ok ? fma(-d, h, 1.0) * h : 0.0;
+}
+
+#ifdef __CUDACC__
+__device__ __noinline__ static double div_division(double x, double d) { return x / d; }
+#endif
+
+// x / d given div_known_prep(d, &yh, &yl, &d_ok).
+__host__ __device__ __forceinline__ double div_known(double x, double d, double yh, double yl, bool d_ok) {
+  const int ex = dexp(x), ed = dexp(d);
+  const bool ok = d_ok && ex >= 64 && ex <= 1983 && ex - ed <= 900 && ed - ex <= 900;
+  const double t = x * yl;
+  double q = fma(x, yh, t);
+  const double r = fma(-q, d, x);
+  q = fma(r, yh, q);
+  if (!ok) {
+#ifdef __CUDA_ARCH__
+    q = div_division(x, d);
+#else
+    q = x / d;
+#endif
+  }
+  return q;
 }
 
 }  // namespace bandlu
