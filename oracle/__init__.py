@@ -67,6 +67,10 @@ def _load():
         lib.oracle_gbtrs.argtypes = [i64, i32, i32, i64, dp, i64, ip, dp, i64]
         lib.oracle_dispatch_lu_batched.argtypes = [dp, i64, i64, i64, i64, dp, i64, i64, ip, i64, ip, ip, ip, ip]
         lib.oracle_dispatch_lu_batched.restype = None
+        lib.oracle_tbsv_dense.argtypes = [i32, i64, i64, dp, i64, i64, dp, i64, ip]
+        lib.oracle_diag_solve.argtypes = [i64, dp, i64, i64, dp, i64, ip]
+        lib.oracle_classify.argtypes = [i64, i32, i32, i64]
+        lib.oracle_dispatch_backslash.argtypes = [dp, i64, i64, dp, i64, i64, dp, i64, ip, ip, ip, ip, ip]
         _lib = lib
         return lib
 
@@ -216,3 +220,62 @@ def dispatch_lu(A: np.ndarray, ldab: int):
     r = dispatch_lu_batched(A[None], ldab)
     return dict(AB=r["AB"][0], ipiv=r["ipiv"][0], kl=int(r["kl"][0]), ku=int(r["ku"][0]),
                 info=int(r["info"][0]), status=int(r["status"][0]))
+
+
+# Kinds of the backslash dispatch (Listing 1), in the order it tests them.
+KIND_DIAGONAL, KIND_LOWER, KIND_UPPER, KIND_BANDED, KIND_DENSE = 1, 2, 3, 4, 5
+
+
+def _rhs(B: np.ndarray, n: int) -> np.ndarray:
+    X = np.array(B, dtype=np.float64, order="C", copy=True)
+    if X.ndim == 1:
+        X = X[None]
+    assert X.shape[1] >= n
+    return X
+
+
+def tbsv_dense(A: np.ndarray, lower: bool, k: int, B: np.ndarray) -> tuple[np.ndarray, int]:
+    """Triangular solve with the band of width k of the (lower or upper) triangle of the
+    row-major A; B (and the result) has shape (nrhs, ldb) as in gbtrs.  Returns (X, info);
+    for info > 0 (a zero diagonal entry) X is B unchanged."""
+    A, n, lda = _dense(A)
+    X = _rhs(B, n)
+    info = ctypes.c_int()
+    rc = _load().oracle_tbsv_dense(1 if lower else 0, n, k, _dptr(A), max(lda, 1), X.shape[0], _dptr(X),
+                                   max(X.shape[1], 1), ctypes.byref(info))
+    if rc != 0:
+        raise ValueError("oracle_tbsv_dense: bad argument")
+    return X, info.value
+
+
+def diag_solve(A: np.ndarray, B: np.ndarray) -> tuple[np.ndarray, int]:
+    """X = B / diag(A) per right-hand side (rows of B); (X, info) as tbsv_dense."""
+    A, n, lda = _dense(A)
+    X = _rhs(B, n)
+    info = ctypes.c_int()
+    rc = _load().oracle_diag_solve(n, _dptr(A), max(lda, 1), X.shape[0], _dptr(X), max(X.shape[1], 1),
+                                   ctypes.byref(info))
+    if rc != 0:
+        raise ValueError("oracle_diag_solve: bad argument")
+    return X, info.value
+
+
+def classify(n: int, kl: int, ku: int, ldab: int) -> int:
+    """The branch of Listing 1 for bandwidths (kl, ku): one of the KIND_* values."""
+    return int(_load().oracle_classify(n, kl, ku, ldab))
+
+
+def dispatch_backslash(A: np.ndarray, B: np.ndarray, ldab: int):
+    """A X = B through the backslash dispatch.  Returns dict with X (nrhs, n), kind, kl, ku,
+    info, and AB, ipiv (the factors, meaningful for KIND_BANDED)."""
+    A, n, lda = _dense(A)
+    X = _rhs(B, n)
+    AB = np.zeros((max(n, 1), ldab), dtype=np.float64)
+    ipiv = np.zeros(max(n, 1), dtype=np.int32)
+    kl, ku, kind, info = ctypes.c_int(), ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    rc = _load().oracle_dispatch_backslash(_dptr(A), n, max(lda, 1), _dptr(X), max(X.shape[1], 1), X.shape[0],
+                                           _dptr(AB), ldab, _iptr(ipiv), ctypes.byref(kl), ctypes.byref(ku),
+                                           ctypes.byref(kind), ctypes.byref(info))
+    if rc != 0:
+        raise ValueError("oracle_dispatch_backslash: bad argument")
+    return dict(X=X, kind=kind.value, kl=kl.value, ku=ku.value, info=info.value, AB=AB[:n], ipiv=ipiv[:n])

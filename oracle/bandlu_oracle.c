@@ -27,6 +27,10 @@
  *   oracle_band_residual      pinned (dense reconstruction with a library matmul)
  *   oracle_is_banded          pinned (the worked cases of the speedup constraint, Eq. su-con)
  *   oracle_gbtrs              pinned (LAPACK dgbtrs; dense solve; exact rational solution; closed form)
+ *   oracle_tbsv_dense         pinned (library triangular solve; exact rational solution; bidiagonal
+ *                             closed form; first-zero-diagonal info)
+ *   oracle_diag_solve         pinned (IEEE quotient by definition; first-zero-diagonal info)
+ *   oracle_classify           pinned (the branch order of Listing 1 on worked cases)
  */
 #include <math.h>
 #include <stdint.h>
@@ -377,5 +381,123 @@ void oracle_dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t
         info[b] = 0;
         status[b] = oracle_dispatch_lu(A + b * strideA, n, lda, AB + b * strideAB, ldab,
                                        ipiv + b * strideP, kl + b, ku + b, info + b);
+    }
+}
+
+/*
+ * Triangular solve on the dense matrix: the LowerTriangular and UpperTriangular
+ * branches of the backslash dispatch (Listing 1, Sec. I-A), taken when the
+ * structure identification finds ku = 0 (istril) or kl = 0 (istriu).  The
+ * triangle has bandwidth k (kl for a lower, ku for an upper one) and only its
+ * band is read.  Semantics of LAPACK xTRTRS: info = the first i (1-based) with
+ * A(i,i) == 0, and then B is left as it is; otherwise every right-hand side
+ * b (a column of B) is overwritten with the solution by the column-oriented
+ * substitution of the reference BLAS (xTBSV, no transpose), with the same
+ * zero test and an fma for each elimination:
+ *   lower, j = 0..n-1:  if b_j != 0:  b_j = b_j / A(j,j);
+ *                                     b_i = fma(-b_j, A(i,j), b_i)  for i = j+1..min(n-1, j+k)
+ *   upper, j = n-1..0:  if b_j != 0:  b_j = b_j / A(j,j);
+ *                                     b_i = fma(-b_j, A(i,j), b_i)  for i = max(0, j-k)..j-1
+ * Returns 0 (info in *info) or -1 on a bad argument.
+ */
+int oracle_tbsv_dense(int lower, int64_t n, int64_t k, const double *A, int64_t lda, int64_t nrhs,
+                      double *B, int64_t ldb, int *info)
+{
+    if (n < 0 || k < 0 || lda < (n > 1 ? n : 1) || nrhs < 0 || ldb < (n > 1 ? n : 1) || !info) return -1;
+    *info = 0;
+    for (int64_t i = 0; i < n; ++i)
+        if (A[i * lda + i] == 0.0) {
+            *info = (int)(i + 1);
+            return 0;
+        }
+    for (int64_t c = 0; c < nrhs; ++c) {
+        double *b = B + c * ldb;
+        if (lower) {
+            for (int64_t j = 0; j < n; ++j) {
+                if (b[j] != 0.0) {
+                    b[j] = b[j] / A[j * lda + j];
+                    const double x = b[j];
+                    const int64_t i1 = j + k < n - 1 ? j + k : n - 1;
+                    for (int64_t i = j + 1; i <= i1; ++i) b[i] = fma(-x, A[i * lda + j], b[i]);
+                }
+            }
+        } else {
+            for (int64_t j = n - 1; j >= 0; --j) {
+                if (b[j] != 0.0) {
+                    b[j] = b[j] / A[j * lda + j];
+                    const double x = b[j];
+                    const int64_t i0 = j - k > 0 ? j - k : 0;
+                    for (int64_t i = i0; i < j; ++i) b[i] = fma(-x, A[i * lda + j], b[i]);
+                }
+            }
+        }
+    }
+    return 0;
+}
+
+/*
+ * Diagonal solve: the Diagonal branch of Listing 1 (Sec. I-A), taken when the
+ * structure identification finds kl = ku = 0.  Diagonal(A) keeps the n diagonal
+ * entries (the memory-efficient format of that branch); the solve divides:
+ * B(i,c) = B(i,c) / A(i,i).  A zero diagonal entry makes the matrix singular:
+ * info = the first such i (1-based) and B is left as it is.
+ * Returns 0 (info in *info) or -1 on a bad argument.
+ */
+int oracle_diag_solve(int64_t n, const double *A, int64_t lda, int64_t nrhs, double *B, int64_t ldb, int *info)
+{
+    if (n < 0 || lda < (n > 1 ? n : 1) || nrhs < 0 || ldb < (n > 1 ? n : 1) || !info) return -1;
+    *info = 0;
+    for (int64_t i = 0; i < n; ++i)
+        if (A[i * lda + i] == 0.0) {
+            *info = (int)(i + 1);
+            return 0;
+        }
+    for (int64_t c = 0; c < nrhs; ++c)
+        for (int64_t i = 0; i < n; ++i) B[c * ldb + i] = B[c * ldb + i] / A[i * lda + i];
+    return 0;
+}
+
+/* Kinds of the backslash dispatch, in the order Listing 1 tests them. */
+enum { ORACLE_KIND_DIAGONAL = 1, ORACLE_KIND_LOWER = 2, ORACLE_KIND_UPPER = 3, ORACLE_KIND_BANDED = 4,
+       ORACLE_KIND_DENSE = 5 };
+
+/*
+ * The branch Listing 1 takes for bandwidths (kl, ku): istril (ku == 0) and
+ * istriu (kl == 0) together give the diagonal solve, istril alone the lower and
+ * istriu alone the upper triangular solve; otherwise LU, through the band path
+ * when the dispatch predicate (oracle_is_banded) accepts it and densely when it
+ * does not.
+ */
+int oracle_classify(int64_t n, int kl, int ku, int64_t ldab)
+{
+    if (ku == 0) return kl == 0 ? ORACLE_KIND_DIAGONAL : ORACLE_KIND_LOWER;
+    if (kl == 0) return ORACLE_KIND_UPPER;
+    return oracle_is_banded(n, kl, ku, ldab) ? ORACLE_KIND_BANDED : ORACLE_KIND_DENSE;
+}
+
+/*
+ * A X = B through the whole backslash dispatch of Listing 1 with the band path
+ * of Sec. II-A: identify (kl, ku), classify, and solve with the branch's
+ * algorithm.  *kind receives the branch.  Diagonal and triangular: the solves
+ * above (info from the zero-diagonal check).  Banded: dispatch_lu, then, when
+ * the factor is nonsingular (info == 0), gbtrs with it.  Dense: nothing is
+ * touched (the caller's dense LU).  Returns 0, or -1 on a bad argument.
+ */
+int oracle_dispatch_backslash(const double *A, int64_t n, int64_t lda, double *B, int64_t ldb, int64_t nrhs,
+                              double *AB, int64_t ldab, int *ipiv, int *kl, int *ku, int *kind, int *info)
+{
+    if (oracle_detect_bandwidth(A, n, lda, kl, ku) != 0) return -1;
+    *info = 0;
+    *kind = oracle_classify(n, *kl, *ku, ldab);
+    switch (*kind) {
+    case ORACLE_KIND_DIAGONAL: return oracle_diag_solve(n, A, lda, nrhs, B, ldb, info);
+    case ORACLE_KIND_LOWER: return oracle_tbsv_dense(1, n, *kl, A, lda, nrhs, B, ldb, info);
+    case ORACLE_KIND_UPPER: return oracle_tbsv_dense(0, n, *ku, A, lda, nrhs, B, ldb, info);
+    case ORACLE_KIND_BANDED:
+        oracle_dense_to_band(A, n, lda, *kl, *ku, AB, ldab);
+        *info = oracle_gbtrf(n, *kl, *ku, AB, ldab, ipiv, 0);
+        if (*info == 0) return oracle_gbtrs(n, *kl, *ku, nrhs, AB, ldab, ipiv, B, ldb);
+        return 0;
+    default: return 0;
     }
 }

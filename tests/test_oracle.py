@@ -552,3 +552,161 @@ def test_gbtrf_ignores_garbage_in_fill_rows(oracle_mod):
     G = AB.copy(); G[:, :kl] = 123.0
     got = oracle_mod.gbtrf(G, kl, ku)
     assert np.array_equal(ref[0], got[0]) and np.array_equal(ref[1], got[1])
+
+
+# ----------------------------------------------------------------------------------------------
+# Triangular and diagonal branches of the backslash dispatch (Listing 1, Sec. I-A)
+# ----------------------------------------------------------------------------------------------
+
+def band_triangle(n, k, lower, seed, boost=2.0, dist="uniform"):
+    """Row-major n x n triangle with bandwidth k (the other triangle zero)."""
+    A = rand_banded(n, k if lower else 0, 0 if lower else k, seed=seed, dist=dist, boost=boost)
+    return A
+
+
+@pytest.mark.parametrize("lower", [True, False])
+def test_tbsv_matches_library_triangular_solve(oracle_mod, lower):
+    """LAPACK's dtrtrs (scipy solve_triangular) on the same triangle: the same solution to rounding."""
+    for idx, (n, k) in enumerate([(1, 0), (2, 1), (9, 3), (64, 16), (150, 40), (120, 119)]):
+        A = band_triangle(n, k, lower, seed=700 + idx, boost=3.0)
+        B = np.random.default_rng(idx).standard_normal((3, n))
+        X, info = oracle_mod.tbsv_dense(A, lower, k, B)
+        assert info == 0
+        ref = scipy.linalg.solve_triangular(A, B.T, lower=lower, check_finite=False).T
+        assert np.max(np.abs(X - ref)) <= 1e-12 * max(np.max(np.abs(ref)), 1.0), (n, k, lower)
+
+
+@pytest.mark.parametrize("lower", [True, False])
+def test_tbsv_exact_rational_solutions(oracle_mod, lower):
+    """Integer triangles with power-of-two diagonals and small integer right-hand sides: every
+    intermediate value is an exact binary fraction, so the oracle must return the rational
+    solution exactly."""
+    rng = np.random.default_rng(11 if lower else 12)
+    for trial in range(60):
+        n, k = int(rng.integers(1, 10)), int(rng.integers(0, 4))
+        A = np.zeros((n, n))
+        for i in range(n):
+            for j in range(n):
+                if (lower and 0 < i - j <= k) or (not lower and 0 < j - i <= k):
+                    A[i, j] = float(rng.integers(-3, 4))
+            A[i, i] = float(2 ** int(rng.integers(0, 3))) * (1 if rng.random() < 0.5 else -1)
+        b = rng.integers(-9, 10, n).astype(float)
+        Af = [[Fraction(int(A[i, j])) for j in range(n)] for i in range(n)]
+        x = [Fraction(int(v)) for v in b]
+        order = range(n) if lower else range(n - 1, -1, -1)
+        for j in order:  # textbook substitution in rationals
+            x[j] = x[j] / Af[j][j]
+            for i in range(n):
+                if (lower and i > j) or (not lower and i < j):
+                    x[i] -= Af[i][j] * x[j]
+        assert all(float(v) == v for v in x)  # exactly representable
+        X, info = oracle_mod.tbsv_dense(A, lower, k, b)
+        assert info == 0
+        assert [Fraction(v) for v in X[0]] == x, (trial, n, k)
+
+
+def test_tbsv_bidiagonal_closed_form(oracle_mod):
+    """Unit bidiagonal with -1 next to the diagonal: the solution is the running sum of b
+    (prefix sums for the lower, suffix sums for the upper triangle), exact in integers."""
+    n = 200
+    b = np.random.default_rng(3).integers(-50, 51, n).astype(float)
+    L = np.eye(n) - np.eye(n, k=-1)
+    X, info = oracle_mod.tbsv_dense(L, True, 1, b)
+    assert info == 0 and np.array_equal(X[0], np.cumsum(b))
+    U = np.eye(n) - np.eye(n, k=1)
+    X, info = oracle_mod.tbsv_dense(U, False, 1, b)
+    assert info == 0 and np.array_equal(X[0], np.cumsum(b[::-1])[::-1])
+
+
+@pytest.mark.parametrize("lower", [True, False])
+def test_tbsv_zero_diagonal_sets_info_and_leaves_b(oracle_mod, lower):
+    """xTRTRS: the first exact zero on the diagonal is reported (1-based) and B is untouched."""
+    n, k = 30, 4
+    A = band_triangle(n, k, lower, seed=5)
+    A[17, 17] = 0.0
+    A[23, 23] = -0.0
+    B = np.random.default_rng(1).standard_normal((2, n))
+    X, info = oracle_mod.tbsv_dense(A, lower, k, B)
+    assert info == 18
+    assert np.array_equal(X, B)
+
+
+@pytest.mark.parametrize("lower", [True, False])
+def test_tbsv_reads_only_its_band(oracle_mod, lower):
+    """Entries outside the triangle's band (NaN here) are never read; an exact zero in b is
+    neither divided nor used (a -0.0 stays -0.0)."""
+    n, k = 40, 3
+    A = band_triangle(n, k, lower, seed=9)
+    G = A.copy()
+    for i in range(n):
+        for j in range(n):
+            if (lower and not 0 <= i - j <= k) or (not lower and not 0 <= j - i <= k):
+                G[i, j] = np.nan
+    b = np.random.default_rng(2).standard_normal(n)
+    X1, _ = oracle_mod.tbsv_dense(A, lower, k, b)
+    X2, _ = oracle_mod.tbsv_dense(G, lower, k, b)
+    assert np.array_equal(X1.view(np.int64), X2.view(np.int64))
+    z = np.zeros(n)
+    z[0 if not lower else n - 1] = -0.0
+    X, _ = oracle_mod.tbsv_dense(A, lower, k, -z)
+    assert np.array_equal(X.view(np.int64), (-z)[None].view(np.int64))
+
+
+def test_diag_solve_is_the_ieee_quotient(oracle_mod):
+    """Diagonal(A) \\ B divides each row by its diagonal entry: numpy's division bit for bit;
+    a zero diagonal entry is reported and leaves B untouched."""
+    rng = np.random.default_rng(4)
+    n = 300
+    d = rng.standard_normal(n) * np.exp(rng.uniform(-30, 30, n))
+    A = np.diag(d)
+    B = rng.standard_normal((4, n))
+    X, info = oracle_mod.diag_solve(A, B)
+    assert info == 0
+    assert np.array_equal(X.view(np.int64), (B / d).view(np.int64))
+    A[100, 100] = 0.0
+    X, info = oracle_mod.diag_solve(A, B)
+    assert info == 101 and np.array_equal(X, B)
+
+
+def test_classify_follows_the_order_of_listing_1(oracle_mod):
+    """istril and istriu: diagonal; istril: lower; istriu: upper; otherwise LU (band path when
+    the dispatch predicate accepts, dense otherwise).  Worked cases of each branch."""
+    K = oracle_mod
+    assert K.classify(100, 0, 0, 1) == K.KIND_DIAGONAL
+    assert K.classify(100, 5, 0, 1) == K.KIND_LOWER  # triangles need no band storage
+    assert K.classify(100, 0, 7, 1) == K.KIND_UPPER
+    assert K.classify(100, 99, 0, 1) == K.KIND_LOWER  # a full triangle too
+    assert K.classify(100, 3, 2, 9) == K.KIND_BANDED
+    assert K.classify(100, 3, 2, 8) == K.KIND_DENSE  # no room for the band
+    assert K.classify(10, 8, 8, 100) == K.KIND_DENSE  # the predicate declines
+    assert K.classify(1, 0, 0, 1) == K.KIND_DIAGONAL
+    for kl, ku in itertools.product(range(4), range(4)):
+        A = rand_banded(12, kl, ku, seed=kl * 4 + ku, boost=4.0)
+        got = K.dispatch_backslash(A, np.ones(12), 2 * kl + ku + 1)
+        assert got["kind"] == K.classify(12, kl, ku, 2 * kl + ku + 1)
+        assert (got["kl"], got["ku"]) == (kl, ku)
+
+
+def test_dispatch_backslash_runs_the_chosen_branch(oracle_mod):
+    """Each kind's solution is that branch's own solve; the dense kind leaves B untouched."""
+    K = oracle_mod
+    rng = np.random.default_rng(8)
+    n = 40
+    B = rng.standard_normal((2, n))
+    D = np.diag(rng.uniform(1, 2, n))
+    r = K.dispatch_backslash(D, B, 1)
+    assert r["kind"] == K.KIND_DIAGONAL and np.array_equal(r["X"], K.diag_solve(D, B)[0])
+    L = band_triangle(n, 5, True, seed=1)
+    r = K.dispatch_backslash(L, B, 1)
+    assert r["kind"] == K.KIND_LOWER and np.array_equal(r["X"], K.tbsv_dense(L, True, 5, B)[0])
+    U = band_triangle(n, 6, False, seed=2)
+    r = K.dispatch_backslash(U, B, 1)
+    assert r["kind"] == K.KIND_UPPER and np.array_equal(r["X"], K.tbsv_dense(U, False, 6, B)[0])
+    A = rand_banded(n, 3, 4, seed=3)
+    r = K.dispatch_backslash(A, B, 11)
+    ABf, ipiv, info, _ = K.gbtrf(K.dense_to_band(A, 3, 4), 3, 4)
+    assert r["kind"] == K.KIND_BANDED and r["info"] == info == 0
+    assert np.array_equal(r["X"], K.gbtrs(ABf, ipiv, 3, 4, B))
+    r = K.dispatch_backslash(A, B, 10)
+    assert r["kind"] == K.KIND_DENSE and np.array_equal(r["X"], B)
+    assert np.max(np.abs(A @ K.dispatch_backslash(A, B, 11)["X"][0] - B[0])) < 1e-10

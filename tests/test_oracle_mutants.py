@@ -44,6 +44,20 @@ MUTANTS = [
     ("gbtrs_update_sign", "b[j + t] = fma(-AB_(kv + t, j), bj, b[j + t]);", "b[j + t] = fma(AB_(kv + t, j), bj, b[j + t]);"),
     ("gbtrs_drops_last_multiplier", "for (int64_t t = 1; t <= km; ++t) b[j + t]", "for (int64_t t = 1; t < km; ++t) b[j + t]"),
     ("gbtrs_drops_top_superdiagonal", "const int64_t i0 = j - kv > 0 ? j - kv : 0;", "const int64_t i0 = j - kv + 1 > 0 ? j - kv + 1 : 0;"),
+    ("tbsv_lower_drops_last_band_entry", "const int64_t i1 = j + k < n - 1 ? j + k : n - 1;",
+     "const int64_t i1 = j + k - 1 < n - 1 ? j + k - 1 : n - 1;"),
+    ("tbsv_upper_update_sign", "for (int64_t i = i0; i < j; ++i) b[i] = fma(-x, A[i * lda + j], b[i]);",
+     "for (int64_t i = i0; i < j; ++i) b[i] = fma(x, A[i * lda + j], b[i]);"),
+    ("tbsv_lower_transposed_operand", "for (int64_t i = j + 1; i <= i1; ++i) b[i] = fma(-x, A[i * lda + j], b[i]);",
+     "for (int64_t i = j + 1; i <= i1; ++i) b[i] = fma(-x, A[j * lda + i], b[i]);"),
+    ("tbsv_lower_skips_division", "b[j] = b[j] / A[j * lda + j];\n                    const double x = b[j];\n                    const int64_t i1",
+     "const double x = b[j];\n                    const int64_t i1"),
+    ("tbsv_info_reports_last_zero", "*info = (int)(i + 1);\n            return 0;\n        }\n    for (int64_t c = 0; c < nrhs; ++c) {\n        double *b",
+     "*info = (int)(i + 1);\n        }\n    for (int64_t c = 0; c < nrhs; ++c) {\n        double *b"),
+    ("diag_multiplies_by_reciprocal", "B[c * ldb + i] = B[c * ldb + i] / A[i * lda + i];",
+     "B[c * ldb + i] = B[c * ldb + i] * (1.0 / A[i * lda + i]);"),
+    ("classify_lower_upper_swapped", "if (ku == 0) return kl == 0 ? ORACLE_KIND_DIAGONAL : ORACLE_KIND_LOWER;",
+     "if (ku == 0) return kl == 0 ? ORACLE_KIND_DIAGONAL : ORACLE_KIND_UPPER;"),
 ]
 
 
