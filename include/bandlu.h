@@ -48,6 +48,14 @@ extern "C" {
 /* dispatch_lu_noalloc: the call would need more scratch than its static array holds */
 #define BANDLU_ERR_SCRATCH 1002
 
+/* Branches of the backslash dispatch (Listing 1, Sec. I-A), in the order it
+ * tests them: bandlu_classify and dispatch_backslash report one of these. */
+#define BANDLU_KIND_DIAGONAL 1 /* kl == 0 and ku == 0 (istril and istriu) */
+#define BANDLU_KIND_LOWER 2    /* ku == 0: lower triangle of bandwidth kl (istril) */
+#define BANDLU_KIND_UPPER 3    /* kl == 0: upper triangle of bandwidth ku (istriu) */
+#define BANDLU_KIND_BANDED 4   /* LU through the band path: the dispatch predicate holds */
+#define BANDLU_KIND_DENSE 5    /* LU the dense way: left to the caller */
+
 /*
  * detect_bandwidth -- structure identification, step 1 of Sec. II-A; cost
  * I(N) ~ O(N^2) (Sec. III-A, Eq. IC-N2); banded_structure(A) in Listing 2.
@@ -154,6 +162,67 @@ int gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t lda
  */
 int dispatch_solve(const double *A, int64_t n, int64_t lda, double *B, int64_t ldb, int64_t nrhs, double *AB,
                    int64_t ldab, int *ipiv, int *h_kl, int *h_ku, int *d_info, cudaStream_t stream);
+
+/*
+ * trsv_band -- the LowerTriangular / UpperTriangular solve of the backslash
+ * dispatch (Listing 1, Sec. I-A), on a triangle of bandwidth k read in place
+ * from the dense ROW-major A (no format conversion; only the band is read).
+ * xTRTRS semantics: *d_info = the first i (1-based) with A(i,i) == 0 and then B
+ * is left as it is, else 0 and every column b of B is overwritten with the
+ * solution by the column-oriented substitution of the reference BLAS (xTBSV, no
+ * transpose), with its zero test and one fma per elimination:
+ *   lower, j = 0..n-1:  if b_j != 0:  b_j = b_j / A(j,j);  b_i = fma(-b_j, A(i,j), b_i), i = j+1..min(n-1, j+k)
+ *   upper, j = n-1..0:  if b_j != 0:  b_j = b_j / A(j,j);  b_i = fma(-b_j, A(i,j), b_i), i = max(0, j-k)..j-1
+ * Arguments: 1 lower (1 = lower, 0 = upper triangle), 2 n >= 0, 3 k (0 <= k <=
+ * max(0, n-1)), 4 A, 5 lda >= max(1, n), 6 B (COLUMN-major n x nrhs, DEVICE),
+ * 7 ldb >= max(1, n), 8 nrhs >= 0, 9 d_info (DEVICE, always written).
+ * Returns BANDLU_OK, -i for a bad argument i, BANDLU_ERR_CUDA.  Asynchronous.
+ * Scratch: none.
+ */
+int trsv_band(int lower, int64_t n, int k, const double *A, int64_t lda, double *B, int64_t ldb, int64_t nrhs,
+              int *d_info, cudaStream_t stream);
+
+/*
+ * diag_solve -- the Diagonal solve of the backslash dispatch (Listing 1): B(i,c)
+ * = B(i,c) / A(i,i) (IEEE division), with A dense ROW-major and only its
+ * diagonal read.  *d_info = the first i (1-based) with A(i,i) == 0 (then B is
+ * left as it is), else 0.
+ * Arguments: 1 n >= 0, 2 A, 3 lda >= max(1, n), 4 B (COLUMN-major n x nrhs),
+ * 5 ldb >= max(1, n), 6 nrhs >= 0, 7 d_info (DEVICE, always written).
+ * Returns BANDLU_OK, -i for a bad argument i, BANDLU_ERR_CUDA.  Asynchronous.
+ */
+int diag_solve(int64_t n, const double *A, int64_t lda, double *B, int64_t ldb, int64_t nrhs, int *d_info,
+               cudaStream_t stream);
+
+/*
+ * bandlu_classify -- the branch Listing 1 takes for detected bandwidths (kl, ku)
+ * (host only, no GPU work): BANDLU_KIND_DIAGONAL when kl == ku == 0, LOWER when
+ * ku == 0, UPPER when kl == 0, otherwise BANDED when the dispatch predicate of
+ * dispatch_lu holds for capacity ldab and DENSE when it does not.  Returns -1
+ * for n < 0, kl < 0 or ku < 0.
+ */
+int bandlu_classify(int64_t n, int kl, int ku, int64_t ldab);
+
+/*
+ * dispatch_backslash -- A X = B through the backslash dispatch of Listing 1
+ * (Sec. I-A) with the band path of Sec. II-A: detect_bandwidth, (kl, ku) read
+ * back to the host (the call waits for `stream` once), bandlu_classify, then
+ * the branch's solve enqueued on `stream`:
+ *   DIAGONAL: diag_solve;  LOWER: trsv_band(1, n, kl);  UPPER: trsv_band(0, n, ku);
+ *   BANDED: dense_to_band, gbtrf and gbtrs with AB and ipiv (the solve is
+ *           skipped on the device when the factor is singular, as in dispatch_solve);
+ *   DENSE: nothing is enqueued and B is untouched (the caller's dense LU).
+ * *d_info is written by every branch but DENSE (first zero diagonal entry, or
+ * gbtrf's info).  *h_kl, *h_ku and *h_kind (HOST) are always written.
+ * Returns BANDLU_OK, BANDLU_NOT_BANDED (the DENSE branch), -i for a bad
+ * argument i, or an error code.
+ * Arguments: 1 A, 2 n, 3 lda, 4 B (COLUMN-major n x nrhs), 5 ldb >= max(1, n),
+ * 6 nrhs >= 0, 7 AB, 8 ldab >= 1, 9 ipiv, 10 h_kl, 11 h_ku, 12 h_kind (HOST),
+ * 13 d_info.  AB and ipiv are only written by the BANDED branch.
+ * Scratch: as dispatch_lu.
+ */
+int dispatch_backslash(const double *A, int64_t n, int64_t lda, double *B, int64_t ldb, int64_t nrhs, double *AB,
+                       int64_t ldab, int *ipiv, int *h_kl, int *h_ku, int *h_kind, int *d_info, cudaStream_t stream);
 
 /*
  * dispatch_lu_batched -- the strategy of Sec. II-A applied to `batch`

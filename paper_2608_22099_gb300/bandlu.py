@@ -59,9 +59,13 @@ def load():
         lib.dispatch_lu_batched.argtypes = [vp, i64, i64, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
         lib.gbtrs.argtypes = [i64, i32, i32, i64, vp, i64, vp, vp, i64, vp]
         lib.dispatch_solve.argtypes = [vp, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
+        lib.trsv_band.argtypes = [i32, i64, i32, vp, i64, vp, i64, i64, vp, vp]
+        lib.diag_solve.argtypes = [i64, vp, i64, vp, i64, i64, vp, vp]
+        lib.bandlu_classify.argtypes = [i64, i32, i32, i64]
+        lib.dispatch_backslash.argtypes = [vp, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp, vp]
         for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "gbtrs", "dispatch_lu", "dispatch_solve",
-                  "dispatch_lu_batched",
-                  "dispatch_lu_noalloc"):
+                  "dispatch_lu_batched", "dispatch_lu_noalloc", "trsv_band", "diag_solve", "bandlu_classify",
+                  "dispatch_backslash"):
             getattr(lib, f).restype = ctypes.c_int
         lib.bandlu_selftest_rcp_host.argtypes = [vp, vp, i64]
         lib.bandlu_selftest_rcp_host.restype = None
@@ -129,6 +133,33 @@ def dispatch_solve(A, n: int, lda: int, B, ldb: int, nrhs: int, AB, ldab: int, i
     rc = load().dispatch_solve(_ptr(A), n, lda, _ptr(B), ldb, nrhs, _ptr(AB), ldab, _ptr(ipiv),
                                ctypes.addressof(kl), ctypes.addressof(ku), _ptr(d_info), _stream(stream))
     return rc, kl.value, ku.value
+
+
+# Branches of the backslash dispatch (BANDLU_KIND_* of bandlu.h).
+KIND_DIAGONAL, KIND_LOWER, KIND_UPPER, KIND_BANDED, KIND_DENSE = 1, 2, 3, 4, 5
+
+
+def trsv_band(lower: int, n: int, k: int, A, lda: int, B, ldb: int, nrhs: int, d_info, stream=None) -> int:
+    return load().trsv_band(lower, n, k, _ptr(A), lda, _ptr(B), ldb, nrhs, _ptr(d_info), _stream(stream))
+
+
+def diag_solve(n: int, A, lda: int, B, ldb: int, nrhs: int, d_info, stream=None) -> int:
+    return load().diag_solve(n, _ptr(A), lda, _ptr(B), ldb, nrhs, _ptr(d_info), _stream(stream))
+
+
+def bandlu_classify(n: int, kl: int, ku: int, ldab: int) -> int:
+    """The branch of the backslash dispatch for bandwidths (kl, ku) (host logic, no GPU work)."""
+    return load().bandlu_classify(n, kl, ku, ldab)
+
+
+def dispatch_backslash(A, n: int, lda: int, B, ldb: int, nrhs: int, AB, ldab: int, ipiv, d_info,
+                       stream=None) -> tuple[int, int, int, int]:
+    """Returns (status, kind, kl, ku); kind, kl and ku are the host outputs of the C call."""
+    kl, ku, kind = ctypes.c_int(-1), ctypes.c_int(-1), ctypes.c_int(-1)
+    rc = load().dispatch_backslash(_ptr(A), n, lda, _ptr(B), ldb, nrhs, _ptr(AB), ldab, _ptr(ipiv),
+                                   ctypes.addressof(kl), ctypes.addressof(ku), ctypes.addressof(kind),
+                                   _ptr(d_info), _stream(stream))
+    return rc, kind.value, kl.value, ku.value
 
 
 def dispatch_lu_noalloc(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -> tuple[int, int, int]:

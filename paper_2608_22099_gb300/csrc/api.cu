@@ -1,5 +1,6 @@
 // api.cu -- the C ABI (declared in include/bandlu.h): argument checks, then the
-// launches of detect.cu, convert.cu, gbtrf.cu, gbtrf_wide.cu, gbtrs.cu and batched.cu.
+// launches of detect.cu, convert.cu, gbtrf.cu, gbtrf_wide.cu, gbtrs.cu,
+// trsolve.cu and batched.cu.
 #include <climits>
 
 #include "common.cuh"
@@ -110,6 +111,89 @@ int dispatch_solve(const double *A, int64_t n, int64_t lda, double *B, int64_t l
   if (rc != BANDLU_OK) return rc;  // BANDLU_NOT_BANDED: B untouched, the caller solves densely
   // the solve reads info on the device and leaves B as it is for a singular factor
   return bandlu::launch_gbtrs(n, *h_kl, *h_ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, stream);
+}
+
+int trsv_band(int lower, int64_t n, int k, const double *A, int64_t lda, double *B, int64_t ldb, int64_t nrhs,
+              int *d_info, cudaStream_t stream) {
+  const bool work = n > 0 && nrhs > 0;
+  if (lower != 0 && lower != 1) return -1;
+  if (bad_n(n)) return -2;
+  if (k < 0 || (n > 0 && k > n - 1)) return -3;
+  if (A == nullptr && n > 0) return -4;
+  if (lda < max1(n)) return -5;
+  if (B == nullptr && work) return -6;
+  if (ldb < max1(n)) return -7;
+  if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -8;
+  if (d_info == nullptr) return -9;
+  return bandlu::launch_trsv(lower == 1, n, k, A, lda, B, ldb, nrhs, d_info, stream);
+}
+
+int diag_solve(int64_t n, const double *A, int64_t lda, double *B, int64_t ldb, int64_t nrhs, int *d_info,
+               cudaStream_t stream) {
+  const bool work = n > 0 && nrhs > 0;
+  if (bad_n(n)) return -1;
+  if (A == nullptr && n > 0) return -2;
+  if (lda < max1(n)) return -3;
+  if (B == nullptr && work) return -4;
+  if (ldb < max1(n)) return -5;
+  if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -6;
+  if (d_info == nullptr) return -7;
+  return bandlu::launch_diag_solve(n, A, lda, B, ldb, nrhs, d_info, stream);
+}
+
+int bandlu_classify(int64_t n, int kl, int ku, int64_t ldab) {
+  if (n < 0 || kl < 0 || ku < 0) return -1;
+  if (ku == 0) return kl == 0 ? BANDLU_KIND_DIAGONAL : BANDLU_KIND_LOWER;
+  if (kl == 0) return BANDLU_KIND_UPPER;
+  return bandlu::predicate_banded(n, kl, ku, ldab) ? BANDLU_KIND_BANDED : BANDLU_KIND_DENSE;
+}
+
+int dispatch_backslash(const double *A, int64_t n, int64_t lda, double *B, int64_t ldb, int64_t nrhs, double *AB,
+                       int64_t ldab, int *ipiv, int *h_kl, int *h_ku, int *h_kind, int *d_info, cudaStream_t stream) {
+  const bool work = n > 0 && nrhs > 0;
+  if (A == nullptr && n > 0) return -1;
+  if (bad_n(n)) return -2;
+  if (lda < max1(n)) return -3;
+  if (B == nullptr && work) return -4;
+  if (ldb < max1(n)) return -5;
+  if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -6;
+  if (AB == nullptr && n > 0) return -7;
+  if (ldab < 1) return -8;
+  if (ipiv == nullptr && n > 0) return -9;
+  if (h_kl == nullptr) return -10;
+  if (h_ku == nullptr) return -11;
+  if (h_kind == nullptr) return -12;
+  if (d_info == nullptr) return -13;
+  int *d_klku = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&d_klku), 2 * sizeof(int), stream) != cudaSuccess)
+    return BANDLU_ERR_CUDA;
+  int rc = bandlu::launch_detect(A, n, lda, d_klku, d_klku + 1, stream);
+  int h[2] = {0, 0};
+  if (rc == BANDLU_OK && cudaMemcpyAsync(h, d_klku, sizeof(h), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    rc = BANDLU_ERR_CUDA;
+  if (cudaFreeAsync(d_klku, stream) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (cudaStreamSynchronize(stream) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (rc != BANDLU_OK) return rc;
+  const int kl = h[0], ku = h[1];
+  *h_kl = kl;
+  *h_ku = ku;
+  const int kind = bandlu_classify(n, kl, ku, ldab);
+  *h_kind = kind;
+  switch (kind) {
+    case BANDLU_KIND_DIAGONAL:
+      return bandlu::launch_diag_solve(n, A, lda, B, ldb, nrhs, d_info, stream);
+    case BANDLU_KIND_LOWER:
+      return bandlu::launch_trsv(true, n, kl, A, lda, B, ldb, nrhs, d_info, stream);
+    case BANDLU_KIND_UPPER:
+      return bandlu::launch_trsv(false, n, ku, A, lda, B, ldb, nrhs, d_info, stream);
+    case BANDLU_KIND_BANDED:
+      rc = bandlu::launch_dense_to_band(A, lda, n, kl, ku, AB, ldab, stream);
+      if (rc == BANDLU_OK) rc = bandlu::launch_gbtrf(n, kl, ku, AB, ldab, ipiv, d_info, stream);
+      if (rc == BANDLU_OK) rc = bandlu::launch_gbtrs(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, d_info, stream);
+      return rc;
+    default:
+      return BANDLU_NOT_BANDED;  // B untouched: the caller's dense LU
+  }
 }
 
 int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,

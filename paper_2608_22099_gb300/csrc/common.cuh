@@ -120,6 +120,12 @@ int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *
 // d_info: when not null and *d_info != 0 (a singular factor), B is left as it is.
 int launch_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
                  int64_t ldb, const int *d_info, cudaStream_t s);
+// Triangular solve with the band of width k of A's lower (or upper) triangle,
+// and the diagonal solve; both write *d_info (first zero diagonal entry).
+int launch_trsv(bool lower, int64_t n, int k, const double *A, int64_t lda, double *B, int64_t ldb, int64_t nrhs,
+                int *d_info, cudaStream_t s);
+int launch_diag_solve(int64_t n, const double *A, int64_t lda, double *B, int64_t ldb, int64_t nrhs, int *d_info,
+                      cudaStream_t s);
 int launch_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int64_t batch, double *AB,
                    int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP, int *d_kl, int *d_ku, int *d_info,
                    int *d_status, cudaStream_t s);

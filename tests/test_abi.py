@@ -142,3 +142,60 @@ def test_binding_has_the_c_names():
         if name == "bandlu_version":
             continue
         assert callable(getattr(bandlu, name)), name
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((2, 4, 1, DEV, 4, DEV, 4, 1, DEV), -1),
+    ((1, -1, 1, DEV, 4, DEV, 4, 1, DEV), -2),
+    ((1, 4, -1, DEV, 4, DEV, 4, 1, DEV), -3),
+    ((1, 4, 4, DEV, 4, DEV, 4, 1, DEV), -3),
+    ((1, 4, 1, 0, 4, DEV, 4, 1, DEV), -4),
+    ((0, 4, 1, DEV, 3, DEV, 4, 1, DEV), -5),
+    ((1, 4, 1, DEV, 4, 0, 4, 1, DEV), -6),
+    ((1, 4, 1, DEV, 4, DEV, 3, 1, DEV), -7),
+    ((1, 4, 1, DEV, 4, DEV, 4, -1, DEV), -8),
+    ((1, 4, 1, DEV, 4, DEV, 4, 1, 0), -9),
+])
+def test_trsv_band_argument_checks(args, expect):
+    assert bandlu.trsv_band(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((-1, DEV, 4, DEV, 4, 1, DEV), -1),
+    ((4, 0, 4, DEV, 4, 1, DEV), -2),
+    ((4, DEV, 3, DEV, 4, 1, DEV), -3),
+    ((4, DEV, 4, 0, 4, 1, DEV), -4),
+    ((4, DEV, 4, DEV, 3, 1, DEV), -5),
+    ((4, DEV, 4, DEV, 4, -1, DEV), -6),
+    ((4, DEV, 4, DEV, 4, 1, 0), -7),
+])
+def test_diag_solve_argument_checks(args, expect):
+    assert bandlu.diag_solve(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, DEV, 4, 1, DEV, 4, DEV, DEV), -1),
+    ((DEV, -2, 4, DEV, 4, 1, DEV, 4, DEV, DEV), -2),
+    ((DEV, 4, 3, DEV, 4, 1, DEV, 4, DEV, DEV), -3),
+    ((DEV, 4, 4, 0, 4, 1, DEV, 4, DEV, DEV), -4),
+    ((DEV, 4, 4, DEV, 3, 1, DEV, 4, DEV, DEV), -5),
+    ((DEV, 4, 4, DEV, 4, -1, DEV, 4, DEV, DEV), -6),
+    ((DEV, 4, 4, DEV, 4, 1, 0, 4, DEV, DEV), -7),
+    ((DEV, 4, 4, DEV, 4, 1, DEV, 0, DEV, DEV), -8),
+    ((DEV, 4, 4, DEV, 4, 1, DEV, 4, 0, DEV), -9),
+    ((DEV, 4, 4, DEV, 4, 1, DEV, 4, DEV, 0), -13),
+])
+def test_dispatch_backslash_argument_checks(args, expect):
+    rc, _, _, _ = bandlu.dispatch_backslash(*args, stream=0)
+    assert rc == expect
+
+
+def test_classify_matches_the_oracle(oracle_mod):
+    """The host-side branch choice of the backslash dispatch agrees with the oracle's."""
+    import itertools
+    assert bandlu.bandlu_classify(4, -1, 0, 4) == -1
+    for n, kl, ku, ldab in itertools.product([0, 1, 2, 7, 64, 1000, 1 << 20], [0, 1, 3, 30, 999],
+                                             [0, 1, 2, 64, 500], [1, 4, 10, 200, 4000]):
+        if n and (kl > n - 1 or ku > n - 1):
+            continue
+        assert bandlu.bandlu_classify(n, kl, ku, ldab) == oracle_mod.classify(n, kl, ku, ldab), (n, kl, ku, ldab)
