@@ -490,6 +490,24 @@ def run_workload_report(args):
             disp()
         t_disp = timed(disp, reps)
         t_det = timed(det, reps)
+        # the same dispatch with the decision on the device (no host round trip), and that call
+        # captured once in a CUDA graph and replayed
+        sc = torch.zeros(4, dtype=torch.int32, device=dev)
+
+        def dasync(st):
+            bandlu.check(bandlu.dispatch_lu_async(A, n, n, AB, ldab, ipiv, sc[0:1], sc[1:2], sc[2:3], sc[3:4], st),
+                         "dispatch_lu_async")
+        for _ in range(3):
+            dasync(stream)
+        t_async = timed(lambda: dasync(stream), reps)
+        gs = torch.cuda.Stream()
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=gs):
+            dasync(gs)
+        graph.replay()
+        t_graph = timed(graph.replay, reps)
+        out.update({"dispatch_async_ms": t_async * 1e3, "dispatch_graph_ms": t_graph * 1e3})
         rc, dkl, dku = res["rc"]
         out.update({"status": rc, "detected_kl": dkl, "detected_ku": dku, "dispatch_ms": t_disp * 1e3,
                     "detect_us": t_det * 1e6, "detect_gbs": 8.0 * n * n / t_det / 1e9,

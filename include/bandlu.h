@@ -129,6 +129,27 @@ int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t lda
                 int *h_ku, int *d_info, cudaStream_t stream);
 
 /*
+ * dispatch_lu_async -- dispatch_lu with the decision taken on the device: the
+ * same identification, predicate, conversion and factorisation, enqueued on
+ * `stream` without any host synchronisation or allocation, so that a caller can
+ * queue dispatches back to back or capture the call in a CUDA graph.
+ * Outputs, all in DEVICE memory: *d_kl, *d_ku (as detect_bandwidth), *d_status
+ * (BANDLU_OK: factored, *d_info written by the factorisation; BANDLU_NOT_BANDED:
+ * declined, AB, ipiv and *d_info untouched).  The factors are those of
+ * dispatch_lu (the same kernels and order of operations) for every band whose
+ * active window fits a shared-memory window of one CTA (kl <= 27 and
+ * 2*kl+ku+1 <= 256); wider bands are factored by a single CTA column by column
+ * (the same results, more slowly: the multi-CTA kernel dispatch_lu uses there
+ * is sized from kl on the host).
+ * Arguments: 1 A, 2 n, 3 lda, 4 AB, 5 ldab (1 <= ldab < 2^31), 6 ipiv,
+ * 7 d_kl, 8 d_ku, 9 d_status, 10 d_info (DEVICE, distinct).
+ * Returns BANDLU_OK (work enqueued), -i for a bad argument i, BANDLU_ERR_CUDA.
+ * Scratch: none.
+ */
+int dispatch_lu_async(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *d_kl,
+                      int *d_ku, int *d_status, int *d_info, cudaStream_t stream);
+
+/*
  * gbtrs -- the solve after the factorisation: the backslash operator the
  * dispatch of Listing 1 (Sec. I-A) stands for, on the band path (LAPACK xGBTRS,
  * no transpose).  Solves A X = B with A = P0 L0 P1 L1 ... U as left in AB and

@@ -59,12 +59,13 @@ def load():
         lib.dispatch_lu_batched.argtypes = [vp, i64, i64, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
         lib.gbtrs.argtypes = [i64, i32, i32, i64, vp, i64, vp, vp, i64, vp]
         lib.dispatch_solve.argtypes = [vp, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
+        lib.dispatch_lu_async.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp, vp]
         lib.trsv_band.argtypes = [i32, i64, i32, vp, i64, vp, i64, i64, vp, vp]
         lib.diag_solve.argtypes = [i64, vp, i64, vp, i64, i64, vp, vp]
         lib.bandlu_classify.argtypes = [i64, i32, i32, i64]
         lib.dispatch_backslash.argtypes = [vp, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp, vp]
         for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "gbtrs", "dispatch_lu", "dispatch_solve",
-                  "dispatch_lu_batched", "dispatch_lu_noalloc", "trsv_band", "diag_solve", "bandlu_classify",
+                  "dispatch_lu_batched", "dispatch_lu_noalloc", "dispatch_lu_async", "trsv_band", "diag_solve", "bandlu_classify",
                   "dispatch_backslash"):
             getattr(lib, f).restype = ctypes.c_int
         lib.bandlu_selftest_rcp_host.argtypes = [vp, vp, i64]
@@ -120,6 +121,12 @@ def dispatch_lu(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -
     rc = load().dispatch_lu(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), ctypes.addressof(kl),
                             ctypes.addressof(ku), _ptr(d_info), _stream(stream))
     return rc, kl.value, ku.value
+
+
+def dispatch_lu_async(A, n: int, lda: int, AB, ldab: int, ipiv, d_kl, d_ku, d_status, d_info, stream=None) -> int:
+    """dispatch_lu with the decision on the device: no host synchronisation; outputs in device memory."""
+    return load().dispatch_lu_async(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), _ptr(d_kl), _ptr(d_ku),
+                                    _ptr(d_status), _ptr(d_info), _stream(stream))
 
 
 def gbtrs(n: int, kl: int, ku: int, nrhs: int, AB, ldab: int, ipiv, B, ldb: int, stream=None) -> int:

@@ -77,6 +77,24 @@ int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t lda
   return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream);
 }
 
+int dispatch_lu_async(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *d_kl,
+                      int *d_ku, int *d_status, int *d_info, cudaStream_t stream) {
+  if (A == nullptr && n > 0) return -1;
+  if (bad_n(n)) return -2;
+  if (lda < max1(n)) return -3;
+  if (AB == nullptr && n > 0) return -4;
+  if (ldab < 1 || ldab > (int64_t)INT_MAX) return -5;
+  if (ipiv == nullptr && n > 0) return -6;
+  if (d_kl == nullptr) return -7;
+  if (d_ku == nullptr) return -8;
+  if (d_status == nullptr) return -9;
+  if (d_info == nullptr) return -10;
+  int rc = bandlu::launch_detect(A, n, lda, d_kl, d_ku, stream);
+  if (rc == BANDLU_OK) rc = bandlu::launch_decide_convert(A, lda, n, ldab, d_kl, d_ku, d_status, AB, stream);
+  if (rc == BANDLU_OK) rc = bandlu::launch_gbtrf_on_device(n, AB, ldab, ipiv, d_kl, d_ku, d_status, d_info, stream);
+  return rc;
+}
+
 int gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
           int64_t ldb, cudaStream_t stream) {
   const bool work = n > 0 && nrhs > 0;

@@ -117,6 +117,13 @@ int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv,
                  bool allow_alloc = true);
 int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t s,
                       bool *used);
+// dispatch_lu_async: the decision and the conversion with (kl, ku) read on the
+// device (*d_status = BANDLU_OK or BANDLU_NOT_BANDED), then the factorisation
+// it selects (nothing when declined).
+int launch_decide_convert(const double *A, int64_t lda, int64_t n, int64_t ldab, const int *d_kl, const int *d_ku,
+                          int *d_status, double *AB, cudaStream_t s);
+int launch_gbtrf_on_device(int64_t n, double *AB, int64_t ldab, int *ipiv, const int *d_kl, const int *d_ku,
+                           const int *d_status, int *d_info, cudaStream_t s);
 // d_info: when not null and *d_info != 0 (a singular factor), B is left as it is.
 int launch_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
                  int64_t ldb, const int *d_info, cudaStream_t s);

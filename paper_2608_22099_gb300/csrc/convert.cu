@@ -54,7 +54,72 @@ __global__ void __launch_bounds__(256) k_dense_to_band_direct(const double *__re
   }
 }
 
+// dispatch_lu_async: the decision taken on the device.  Every block reads the
+// detected (kl, ku), applies the dispatch predicate (block 0 records it in
+// *d_status) and, for a banded matrix, converts its tile as k_dense_to_band_tiled
+// does (the tile size depends on ldab only).
+__global__ void __launch_bounds__(256) k_decide_convert_tiled(const double *__restrict__ A, long long lda, long long n,
+                                                              const int *__restrict__ d_kl,
+                                                              const int *__restrict__ d_ku, int *__restrict__ d_status,
+                                                              double *__restrict__ AB, long long ldab, int T) {
+  const long long kl = *d_kl, ku = *d_ku;
+  const bool banded = predicate_banded(n, kl, ku, ldab);
+  if (blockIdx.x == 0 && threadIdx.x == 0) *d_status = banded ? BANDLU_OK : BANDLU_NOT_BANDED;
+  if (!banded) return;  // whole block
+  extern __shared__ double tile[];
+  const long long kv = kl + ku;
+  const long long j0 = (long long)blockIdx.x * T;
+  const int tcols = (int)min((long long)T, n - j0);
+  const long long tsize = (long long)tcols * ldab;
+  for (long long e = threadIdx.x; e < tsize; e += blockDim.x) tile[e] = 0.0;
+  __syncthreads();
+  const long long i_lo = max(0ll, j0 - ku);
+  const long long i_hi = min(n - 1, j0 + tcols - 1 + kl);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+  for (long long i = i_lo + warp; i <= i_hi; i += nwarps) {
+    const long long c_lo = max(j0, i - kl);
+    const long long c_hi = min(min(j0 + tcols - 1, i + ku), n - 1);
+    for (long long c = c_lo + lane; c <= c_hi; c += 32) tile[(c - j0) * ldab + (kv + i - c)] = A[i * lda + c];
+  }
+  __syncthreads();
+  double *out = AB + j0 * ldab;
+  for (long long e = threadIdx.x; e < tsize; e += blockDim.x) out[e] = tile[e];
+}
+
+// The direct form of the same, for very tall band storage.
+__global__ void __launch_bounds__(256) k_decide_convert_direct(const double *__restrict__ A, long long lda,
+                                                               long long n, const int *__restrict__ d_kl,
+                                                               const int *__restrict__ d_ku,
+                                                               int *__restrict__ d_status, double *__restrict__ AB,
+                                                               long long ldab) {
+  const long long kl = *d_kl, ku = *d_ku;
+  const bool banded = predicate_banded(n, kl, ku, ldab);
+  if (blockIdx.x == 0 && threadIdx.x == 0) *d_status = banded ? BANDLU_OK : BANDLU_NOT_BANDED;
+  if (!banded) return;
+  const long long kv = kl + ku;
+  const long long total = n * ldab;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long j = e / ldab;
+    const long long r = e - j * ldab;
+    const long long i = j - kv + r;
+    double v = 0.0;
+    if (r >= kl && r <= kv + kl && i >= 0 && i < n) v = A[i * lda + j];
+    AB[e] = v;
+  }
+}
+
 constexpr int kTileSmemMax = 96 * 1024;
+
+// Columns per tile for band storage of height ldab: enough blocks to cover the
+// SMs for small n, at most 32; 0 when one column does not fit the tile.
+int tile_columns(long long n, long long ldab) {
+  const long long per_col = ldab * (long long)sizeof(double);
+  if (per_col > kTileSmemMax) return 0;
+  int T = (int)min(32ll, (long long)kTileSmemMax / per_col);
+  while (T > 1 && (n + T - 1) / T < 304) T >>= 1;
+  return T < 1 ? 1 : T;
+}
 
 }  // namespace
 
@@ -62,11 +127,8 @@ int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku
                          cudaStream_t s) {
   if (n == 0) return BANDLU_OK;
   const long long per_col = ldab * (long long)sizeof(double);
-  if (per_col <= kTileSmemMax) {
-    // T columns per block: enough blocks to cover the SMs for small n, at most 32.
-    int T = (int)min(32ll, (long long)kTileSmemMax / per_col);
-    while (T > 1 && (n + T - 1) / T < 304) T >>= 1;
-    if (T < 1) T = 1;
+  const int T = tile_columns(n, ldab);
+  if (T > 0) {
     const size_t smem = (size_t)T * per_col;
     static bool attr_set = false;
     if (!attr_set) {
@@ -82,6 +144,26 @@ int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku
     long long blocks = (total + 255) / 256;
     if (blocks > 152ll * 32) blocks = 152ll * 32;
     k_dense_to_band_direct<<<(unsigned)blocks, 256, 0, s>>>(A, lda, n, kl, ku, AB, ldab);
+  }
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+int launch_decide_convert(const double *A, int64_t lda, int64_t n, int64_t ldab, const int *d_kl, const int *d_ku,
+                          int *d_status, double *AB, cudaStream_t s) {
+  const int T = n > 0 ? tile_columns(n, ldab) : 0;  // n == 0: the direct kernel records the decision
+  if (T > 0) {
+    const size_t smem = (size_t)T * ldab * sizeof(double);
+    static const bool attr = cudaFuncSetAttribute(k_decide_convert_tiled, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                  kTileSmemMax) == cudaSuccess;
+    if (!attr) return BANDLU_ERR_CUDA;
+    k_decide_convert_tiled<<<(unsigned)((n + T - 1) / T), 256, smem, s>>>(A, lda, n, d_kl, d_ku, d_status, AB, ldab,
+                                                                          T);
+  } else {
+    long long blocks = (n * ldab + 255) / 256;
+    if (blocks > 152ll * 32) blocks = 152ll * 32;
+    if (blocks < 1) blocks = 1;
+    k_decide_convert_direct<<<(unsigned)blocks, 256, 0, s>>>(A, lda, n, d_kl, d_ku, d_status, AB, ldab);
   }
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;

@@ -130,12 +130,12 @@ struct WinShared {
 // pivot chain of the panel warp.
 __device__ __noinline__ double div_slow(double x) { return 1.0 / x; }
 
+// The window factorisation (kWarps warps; W: R * CS doubles of dynamic shared
+// memory), for k_gbtrf_window and the device-side dispatch.
 template <int K, int PF>
-__global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, int ku, double *__restrict__ AB,
-                                                                  long long ldab, int *__restrict__ ipiv,
-                                                                  int *__restrict__ d_info) {
-  extern __shared__ double W[];  // R * CS
-  __shared__ WinShared sh;
+__device__ __forceinline__ void window_factor(int n, int kl, int ku, double *__restrict__ AB, long long ldab,
+                                              int *__restrict__ ipiv, int *__restrict__ d_info, double *W,
+                                              WinShared &sh) {
   const int kv = kl + ku;
   const int R = kl + 1 + kDelta;
   const int CS = kl + kv + 1;
@@ -376,9 +376,19 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, 
   if (threadIdx.x == 0) *d_info = BAR_FAILED() ? -BANDLU_ERR_TIMEOUT : info;
 }
 
-__global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int ku, double *__restrict__ AB,
-                                                         long long ldab, int *__restrict__ ipiv,
-                                                         int *__restrict__ d_info) {
+template <int K, int PF>
+__global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_window(int n, int kl, int ku, double *__restrict__ AB,
+                                                                  long long ldab, int *__restrict__ ipiv,
+                                                                  int *__restrict__ d_info) {
+  extern __shared__ double W[];  // R * CS
+  __shared__ WinShared sh;
+  window_factor<K, PF>(n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+}
+
+// Column-by-column elimination by the whole block (any block size) on AB in
+// global memory, for k_gbtrf_generic and the device-side dispatch.
+__device__ __forceinline__ void generic_factor(long long n, int kl, int ku, double *__restrict__ AB, long long ldab,
+                                               int *__restrict__ ipiv, int *__restrict__ d_info) {
   __shared__ KeyIdx s_red[32];
   __shared__ int s_p;
   __shared__ double s_r;
@@ -445,12 +455,19 @@ __global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int
   if (tid == 0) *d_info = info;
 }
 
+__global__ void __launch_bounds__(1024) k_gbtrf_generic(long long n, int kl, int ku, double *__restrict__ AB,
+                                                         long long ldab, int *__restrict__ ipiv,
+                                                         int *__restrict__ d_info) {
+  generic_factor(n, kl, ku, AB, ldab, ipiv, d_info);
+}
+
 // The narrowest bands, (kl+1)*(kl+ku+1) <= 32: one warp with the active window
 // in registers (regwin.cuh).  Fill-row entries above the matrix are cleared
 // first, as the elimination clears every fill row; the window writes the rest.
-__global__ void __launch_bounds__(32) k_gbtrf_regwin(int n, int kl, int ku, double *__restrict__ AB, int ldab,
-                                                     int *__restrict__ ipiv, int *__restrict__ d_info) {
-  const int kv = kl + ku, lane = threadIdx.x;
+// Called by one whole warp.
+__device__ __forceinline__ void regwin_factor(int n, int kl, int ku, double *__restrict__ AB, int ldab,
+                                              int *__restrict__ ipiv, int *__restrict__ d_info) {
+  const int kv = kl + ku, lane = threadIdx.x & 31;
   if (kl > 0) {
     for (int e = lane; e < kl * min(n, kv); e += 32) {
       const int jj = e / kl, rr = e - jj * kl;
@@ -464,6 +481,74 @@ __global__ void __launch_bounds__(32) k_gbtrf_regwin(int n, int kl, int ku, doub
   int info[1];
   regwin::window_gbtrf<1>(abp, ldab, n, klv, kuv, pvp, info);
   if (lane == 0) *d_info = info[0];
+}
+
+__global__ void __launch_bounds__(32) k_gbtrf_regwin(int n, int kl, int ku, double *__restrict__ AB, int ldab,
+                                                     int *__restrict__ ipiv, int *__restrict__ d_info) {
+  regwin_factor(n, kl, ku, AB, ldab, ipiv, d_info);
+}
+
+// The path choice of launch_gbtrf (without the multi-CTA kernel), shared by the
+// host launcher and the device-side dispatch: 0 register window, 1 shared-
+// memory window (*K, *PF: its template parameters, *smem: its bytes), 2 generic.
+__host__ __device__ inline int factor_path(long long n, int kl, int ku, long long ldab, int *K, int *PF,
+                                           size_t *smem) {
+  const long long kv = (long long)kl + ku;
+  if ((kl + 1LL) * (kv + 1) <= 32 && (n + 1) * ldab < (long long)INT_MAX) return 0;
+  const long long CS = kl + kv + 1;
+  const long long R = kl + 1 + kDelta;
+  *smem = (size_t)(R * CS) * sizeof(double);
+  const long long E = kv > 2 ? (kv - 2) * (kl + 1) : 0;  // trailing elements per step
+  if (kl <= kWinMaxKl && CS <= 8 * 32 && E <= 8 * kNUT && *smem <= 200 * 1024) {
+    const int pf = (int)((CS + 31) / 32);
+    const int k = (int)((E + kNUT - 1) / kNUT);
+    *PF = pf <= 1 ? 1 : (pf <= 2 ? 2 : (pf <= 4 ? 4 : 8));
+    *K = k <= 1 ? 1 : (k <= 2 ? 2 : (k <= 4 ? 4 : 8));
+    return 1;
+  }
+  return 2;
+}
+
+template <int K>
+__device__ __forceinline__ void window_factor_pf(int PF, int n, int kl, int ku, double *AB, long long ldab, int *ipiv,
+                                                 int *d_info, double *W, WinShared &sh) {
+  if (PF == 1) window_factor<K, 1>(n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+  else if (PF == 2) window_factor<K, 2>(n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+  else if (PF == 4) window_factor<K, 4>(n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+  else window_factor<K, 8>(n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+}
+
+// Device-side dispatch: the factorisation of dispatch_lu_async, with (kl, ku)
+// and the dispatch decision read from device memory.  kWarps warps and
+// smem_bytes of dynamic shared memory, enough for every shared-memory window
+// that fits the band storage (2*kl+ku+1 <= ldab); the block takes the path
+// launch_gbtrf would take, except that bands beyond the windows run the
+// block-wide generic elimination (the multi-CTA kernel's grid and scratch are
+// sized from kl on the host).
+__global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_on_device(int n, double *__restrict__ AB, long long ldab,
+                                                                     int *__restrict__ ipiv,
+                                                                     const int *__restrict__ d_kl,
+                                                                     const int *__restrict__ d_ku,
+                                                                     const int *__restrict__ d_status,
+                                                                     int *__restrict__ d_info, size_t smem_bytes) {
+  extern __shared__ double W[];
+  __shared__ WinShared sh;
+  if (*d_status != BANDLU_OK) return;  // declined: nothing is written
+  const int kl = *d_kl, ku = *d_ku;
+  int K = 1, PF = 1;
+  size_t smem = 0;
+  int path = factor_path(n, kl, ku, ldab, &K, &PF, &smem);
+  if (path == 1 && smem > smem_bytes) path = 2;
+  if (path == 0) {
+    if (threadIdx.x < 32) regwin_factor(n, kl, ku, AB, (int)ldab, ipiv, d_info);
+  } else if (path == 1) {
+    if (K == 1) window_factor_pf<1>(PF, n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+    else if (K == 2) window_factor_pf<2>(PF, n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+    else if (K == 4) window_factor_pf<4>(PF, n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+    else window_factor_pf<8>(PF, n, kl, ku, AB, ldab, ipiv, d_info, W, sh);
+  } else {
+    generic_factor(n, kl, ku, AB, ldab, ipiv, d_info);
+  }
 }
 
 template <int K, int PF>
@@ -498,23 +583,19 @@ int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv,
     if (cudaMemsetAsync(d_info, 0, sizeof(int), s) != cudaSuccess) return BANDLU_ERR_CUDA;
     return BANDLU_OK;
   }
-  const long long kv = (long long)kl + ku;
-  if ((kl + 1LL) * (kv + 1) <= 32 && (n + 1) * ldab < (int64_t)INT_MAX) {
+  int K = 1, PF = 1;
+  size_t smem = 0;
+  const int path = factor_path(n, kl, ku, ldab, &K, &PF, &smem);
+  if (path == 0) {
     k_gbtrf_regwin<<<1, 32, 0, s>>>((int)n, kl, ku, AB, (int)ldab, ipiv, d_info);
     BANDLU_CHECK_LAUNCH();
     return BANDLU_OK;
   }
-  const long long CS = kl + kv + 1;
-  const long long R = kl + 1 + kDelta;
-  const size_t smem = (size_t)(R * CS) * sizeof(double);
-  const long long E = kv > 2 ? (kv - 2) * (kl + 1) : 0;  // trailing elements per step
-  if (kl <= kWinMaxKl && CS <= 8 * 32 && E <= 8 * kNUT && smem <= 200 * 1024) {
-    const int pf = (int)((CS + 31) / 32);
-    const int k = (int)((E + kNUT - 1) / kNUT);
-    if (k <= 1) return launch_window_pf<1>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
-    if (k <= 2) return launch_window_pf<2>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
-    if (k <= 4) return launch_window_pf<4>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
-    return launch_window_pf<8>(pf, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+  if (path == 1) {
+    if (K == 1) return launch_window_pf<1>(PF, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+    if (K == 2) return launch_window_pf<2>(PF, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+    if (K == 4) return launch_window_pf<4>(PF, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
+    return launch_window_pf<8>(PF, n, kl, ku, AB, ldab, ipiv, d_info, smem, s);
   }
   if (allow_alloc) {
     bool used = false;
@@ -522,6 +603,26 @@ int launch_gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv,
     if (rc != BANDLU_OK || used) return rc;
   }
   k_gbtrf_generic<<<1, 1024, 0, s>>>(n, kl, ku, AB, ldab, ipiv, d_info);
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+}  // namespace bandlu
+
+namespace bandlu {
+
+int launch_gbtrf_on_device(int64_t n, double *AB, int64_t ldab, int *ipiv, const int *d_kl, const int *d_ku,
+                           const int *d_status, int *d_info, cudaStream_t s) {
+  if (n == 0) return BANDLU_OK;
+  // every shared-memory window that fits the band storage: kl <= kWinMaxKl and
+  // CS = 2*kl+ku+1 <= min(ldab, 256) column slots of R = kl+1+kDelta rows
+  const long long cs = ldab < 256 ? ldab : 256;
+  const size_t smem = (size_t)((kWinMaxKl + 1 + kDelta) * cs) * sizeof(double);
+  static const bool attr =
+      cudaFuncSetAttribute(k_gbtrf_on_device, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) ==
+      cudaSuccess;
+  if (!attr) return BANDLU_ERR_CUDA;
+  k_gbtrf_on_device<<<1, kWarps * 32, smem, s>>>((int)n, AB, ldab, ipiv, d_kl, d_ku, d_status, d_info, smem);
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;
 }

@@ -199,3 +199,19 @@ def test_classify_matches_the_oracle(oracle_mod):
         if n and (kl > n - 1 or ku > n - 1):
             continue
         assert bandlu.bandlu_classify(n, kl, ku, ldab) == oracle_mod.classify(n, kl, ku, ldab), (n, kl, ku, ldab)
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, DEV, 4, DEV, DEV, DEV, DEV, DEV), -1),
+    ((DEV, -2, 4, DEV, 4, DEV, DEV, DEV, DEV, DEV), -2),
+    ((DEV, 4, 3, DEV, 4, DEV, DEV, DEV, DEV, DEV), -3),
+    ((DEV, 4, 4, 0, 4, DEV, DEV, DEV, DEV, DEV), -4),
+    ((DEV, 4, 4, DEV, 0, DEV, DEV, DEV, DEV, DEV), -5),
+    ((DEV, 4, 4, DEV, 4, 0, DEV, DEV, DEV, DEV), -6),
+    ((DEV, 4, 4, DEV, 4, DEV, 0, DEV, DEV, DEV), -7),
+    ((DEV, 4, 4, DEV, 4, DEV, DEV, 0, DEV, DEV), -8),
+    ((DEV, 4, 4, DEV, 4, DEV, DEV, DEV, 0, DEV), -9),
+    ((DEV, 4, 4, DEV, 4, DEV, DEV, DEV, DEV, 0), -10),
+])
+def test_dispatch_lu_async_argument_checks(args, expect):
+    assert bandlu.dispatch_lu_async(*args, stream=0) == expect
