@@ -67,6 +67,8 @@ def _load():
         lib.oracle_gbtrs.argtypes = [i64, i32, i32, i64, dp, i64, ip, dp, i64]
         lib.oracle_dispatch_lu_batched.argtypes = [dp, i64, i64, i64, i64, dp, i64, i64, ip, i64, ip, ip, ip, ip]
         lib.oracle_dispatch_lu_batched.restype = None
+        lib.oracle_detect_bandwidth_cm.argtypes = [dp, i64, i64, ip, ip]
+        lib.oracle_dense_to_band_cm.argtypes = [dp, i64, i64, i32, i32, dp, i64]
         lib.oracle_tbsv_dense.argtypes = [i32, i64, i64, dp, i64, i64, dp, i64, ip]
         lib.oracle_diag_solve.argtypes = [i64, dp, i64, i64, dp, i64, ip]
         lib.oracle_classify.argtypes = [i64, i32, i32, i64]
@@ -279,3 +281,25 @@ def dispatch_backslash(A: np.ndarray, B: np.ndarray, ldab: int):
     if rc != 0:
         raise ValueError("oracle_dispatch_backslash: bad argument")
     return dict(X=X, kind=kind.value, kl=kl.value, ku=ku.value, info=info.value, AB=AB[:n], ipiv=ipiv[:n])
+
+
+def detect_bandwidth_cm(Acm: np.ndarray) -> tuple[int, int]:
+    """(kl, ku) of the n x n matrix stored COLUMN-major: ``Acm`` has shape (n, lda) and
+    ``Acm[j, i]`` is element (i, j) (the row-major array of the transpose)."""
+    Acm, n, lda = _dense(Acm)
+    kl, ku = ctypes.c_int(), ctypes.c_int()
+    rc = _load().oracle_detect_bandwidth_cm(_dptr(Acm), n, max(lda, 1), ctypes.byref(kl), ctypes.byref(ku))
+    if rc != 0:
+        raise ValueError("oracle_detect_bandwidth_cm: bad argument")
+    return kl.value, ku.value
+
+
+def dense_to_band_cm(Acm: np.ndarray, kl: int, ku: int, ldab: int | None = None) -> np.ndarray:
+    """Band storage (n, ldab) of the matrix stored column-major in ``Acm`` (as detect_bandwidth_cm)."""
+    Acm, n, lda = _dense(Acm)
+    ldab = ldab_for(kl, ku) if ldab is None else ldab
+    AB = np.empty((n, ldab), dtype=np.float64)
+    rc = _load().oracle_dense_to_band_cm(_dptr(Acm), n, max(lda, 1), kl, ku, _dptr(AB), ldab)
+    if rc != 0:
+        raise ValueError("oracle_dense_to_band_cm: bad argument")
+    return AB

@@ -31,6 +31,9 @@
  *                             closed form; first-zero-diagonal info)
  *   oracle_diag_solve         pinned (IEEE quotient by definition; first-zero-diagonal info)
  *   oracle_classify           pinned (the branch order of Listing 1 on worked cases)
+ *   oracle_detect_bandwidth_cm, oracle_dense_to_band_cm
+ *                             pinned (the tril/triu characterisation and the row-major conversion
+ *                             of the same matrix)
  */
 #include <math.h>
 #include <stdint.h>
@@ -500,4 +503,40 @@ int oracle_dispatch_backslash(const double *A, int64_t n, int64_t lda, double *B
         return 0;
     default: return 0;
     }
+}
+
+/*
+ * Column-major input (the layout of Julia and LAPACK, which Listing 1 and
+ * Listing 2 operate on): element (i,j) of A is A[i + j*lda].  The same two
+ * definitions as oracle_detect_bandwidth and oracle_dense_to_band, with that
+ * indexing.
+ */
+int oracle_detect_bandwidth_cm(const double *A, int64_t n, int64_t lda, int *kl, int *ku)
+{
+    if (n < 0 || lda < (n > 1 ? n : 1) || !kl || !ku) return -1;
+    int64_t best_l = 0, best_u = 0;
+    for (int64_t j = 0; j < n; ++j) {
+        for (int64_t i = 0; i < n; ++i) {
+            if (is_nonzero(A[i + j * lda])) {
+                if (i - j > best_l) best_l = i - j;
+                if (j - i > best_u) best_u = j - i;
+            }
+        }
+    }
+    *kl = (int)best_l;
+    *ku = (int)best_u;
+    return 0;
+}
+
+int oracle_dense_to_band_cm(const double *A, int64_t n, int64_t lda, int kl, int ku, double *AB, int64_t ldab)
+{
+    if (n < 0 || lda < (n > 1 ? n : 1) || kl < 0 || ku < 0 || ldab < 2 * (int64_t)kl + ku + 1) return -1;
+    const int64_t kv = (int64_t)kl + ku;
+    for (int64_t j = 0; j < n; ++j) {
+        for (int64_t r = 0; r < ldab; ++r) AB[r + j * ldab] = 0.0;
+        const int64_t i0 = j - ku > 0 ? j - ku : 0;
+        const int64_t i1 = j + kl < n - 1 ? j + kl : n - 1;
+        for (int64_t i = i0; i <= i1; ++i) AB[(kv + i - j) + j * ldab] = A[i + j * lda];
+    }
+    return 0;
 }

@@ -710,3 +710,24 @@ def test_dispatch_backslash_runs_the_chosen_branch(oracle_mod):
     r = K.dispatch_backslash(A, B, 10)
     assert r["kind"] == K.KIND_DENSE and np.array_equal(r["X"], B)
     assert np.max(np.abs(A @ K.dispatch_backslash(A, B, 11)["X"][0] - B[0])) < 1e-10
+
+
+# ----------------------------------------------------------------------------------------------
+# Column-major input (the layout Listing 1 and Listing 2 operate on in Julia)
+# ----------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,kl,ku,pad", [(1, 0, 0, 0), (2, 1, 0, 1), (9, 0, 4, 3), (40, 5, 2, 0), (64, 63, 1, 2),
+                                         (100, 7, 30, 5)])
+def test_column_major_detect_and_convert(oracle_mod, n, kl, ku, pad):
+    """Column-major storage of M is the row-major array of M^T (padded rows): detection must give
+    M's bandwidths by the tril/triu characterisation, and the conversion M's band storage as the
+    row-major conversion produces it."""
+    M = rand_banded(n, kl, ku, seed=n + kl + 5 * ku)
+    Acm = np.zeros((n, n + pad))
+    Acm[:, :n] = M.T
+    Acm[:, n:] = np.nan  # padding is never read
+    assert oracle_mod.detect_bandwidth_cm(Acm) == bandwidth_by_tril_triu(M) == (kl, ku)
+    for ldab in (2 * kl + ku + 1, 2 * kl + ku + 4):
+        AB = oracle_mod.dense_to_band_cm(Acm, kl, ku, ldab)
+        assert np.array_equal(AB.view(np.int64), oracle_mod.dense_to_band(M, kl, ku, ldab).view(np.int64))
+        assert np.array_equal(oracle_mod.band_to_dense(AB, kl, ku), M)

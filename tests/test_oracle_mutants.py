@@ -56,6 +56,9 @@ MUTANTS = [
      "*info = (int)(i + 1);\n        }\n    for (int64_t c = 0; c < nrhs; ++c) {\n        double *b"),
     ("diag_multiplies_by_reciprocal", "B[c * ldb + i] = B[c * ldb + i] / A[i * lda + i];",
      "B[c * ldb + i] = B[c * ldb + i] * (1.0 / A[i * lda + i]);"),
+    ("cm_detect_reads_row_major", "if (is_nonzero(A[i + j * lda])) {", "if (is_nonzero(A[j + i * lda])) {"),
+    ("cm_convert_drops_top_superdiagonal", "const int64_t i0 = j - ku > 0 ? j - ku : 0;\n        const int64_t i1 = j + kl < n - 1 ? j + kl : n - 1;\n        for (int64_t i = i0; i <= i1; ++i) AB[(kv + i - j) + j * ldab] = A[i + j * lda];",
+     "const int64_t i0 = j - ku + 1 > 0 ? j - ku + 1 : 0;\n        const int64_t i1 = j + kl < n - 1 ? j + kl : n - 1;\n        for (int64_t i = i0; i <= i1; ++i) AB[(kv + i - j) + j * ldab] = A[i + j * lda];"),
     ("classify_lower_upper_swapped", "if (ku == 0) return kl == 0 ? ORACLE_KIND_DIAGONAL : ORACLE_KIND_LOWER;",
      "if (ku == 0) return kl == 0 ? ORACLE_KIND_DIAGONAL : ORACLE_KIND_UPPER;"),
 ]
