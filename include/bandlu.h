@@ -107,6 +107,17 @@ int dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, doubl
 int gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t stream);
 
 /*
+ * detect_bandwidth_cm, dense_to_band_cm -- detect_bandwidth and dense_to_band
+ * for a COLUMN-major A (the layout of the Julia code the paper's listings are
+ * written in): element (i, j) is A[i + j*lda].  Same definitions, arguments,
+ * outputs and return codes as the row-major calls; A's columns are contiguous,
+ * so the conversion reads each band column in one run.
+ */
+int detect_bandwidth_cm(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t stream);
+int dense_to_band_cm(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                     cudaStream_t stream);
+
+/*
  * dispatch_lu -- the whole strategy of Sec. II-A for one matrix
  * (structure_aware_lu of Listing 2 without the dense branch).
  *
@@ -127,6 +138,14 @@ int gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d
  */
 int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *h_kl,
                 int *h_ku, int *d_info, cudaStream_t stream);
+
+/*
+ * dispatch_lu_cm -- dispatch_lu for a COLUMN-major A (A(i,j) = A[i + j*lda]):
+ * detect_bandwidth_cm, the same predicate, dense_to_band_cm and gbtrf.  Same
+ * arguments, outputs, return codes and scratch as dispatch_lu.
+ */
+int dispatch_lu_cm(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *h_kl,
+                   int *h_ku, int *d_info, cudaStream_t stream);
 
 /*
  * dispatch_lu_async -- dispatch_lu with the decision taken on the device: the

@@ -59,13 +59,17 @@ def load():
         lib.dispatch_lu_batched.argtypes = [vp, i64, i64, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
         lib.gbtrs.argtypes = [i64, i32, i32, i64, vp, i64, vp, vp, i64, vp]
         lib.dispatch_solve.argtypes = [vp, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
+        lib.detect_bandwidth_cm.argtypes = [vp, i64, i64, vp, vp, vp]
+        lib.dense_to_band_cm.argtypes = [vp, i64, i64, i32, i32, vp, i64, vp]
+        lib.dispatch_lu_cm.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp]
         lib.dispatch_lu_async.argtypes = [vp, i64, i64, vp, i64, vp, vp, vp, vp, vp, vp]
         lib.trsv_band.argtypes = [i32, i64, i32, vp, i64, vp, i64, i64, vp, vp]
         lib.diag_solve.argtypes = [i64, vp, i64, vp, i64, i64, vp, vp]
         lib.bandlu_classify.argtypes = [i64, i32, i32, i64]
         lib.dispatch_backslash.argtypes = [vp, i64, i64, vp, i64, i64, vp, i64, vp, vp, vp, vp, vp, vp]
         for f in ("detect_bandwidth", "dense_to_band", "gbtrf", "gbtrs", "dispatch_lu", "dispatch_solve",
-                  "dispatch_lu_batched", "dispatch_lu_noalloc", "dispatch_lu_async", "trsv_band", "diag_solve", "bandlu_classify",
+                  "dispatch_lu_batched", "dispatch_lu_noalloc", "dispatch_lu_async", "trsv_band",
+                  "detect_bandwidth_cm", "dense_to_band_cm", "dispatch_lu_cm", "diag_solve", "bandlu_classify",
                   "dispatch_backslash"):
             getattr(lib, f).restype = ctypes.c_int
         lib.bandlu_selftest_rcp_host.argtypes = [vp, vp, i64]
@@ -120,6 +124,24 @@ def dispatch_lu(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -
     kl, ku = ctypes.c_int(-1), ctypes.c_int(-1)
     rc = load().dispatch_lu(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), ctypes.addressof(kl),
                             ctypes.addressof(ku), _ptr(d_info), _stream(stream))
+    return rc, kl.value, ku.value
+
+
+def detect_bandwidth_cm(A, n: int, lda: int, d_kl, d_ku, stream=None) -> int:
+    """detect_bandwidth for a column-major A (element (i, j) at A[i + j*lda])."""
+    return load().detect_bandwidth_cm(_ptr(A), n, lda, _ptr(d_kl), _ptr(d_ku), _stream(stream))
+
+
+def dense_to_band_cm(A, lda: int, n: int, kl: int, ku: int, AB, ldab: int, stream=None) -> int:
+    """dense_to_band for a column-major A."""
+    return load().dense_to_band_cm(_ptr(A), lda, n, kl, ku, _ptr(AB), ldab, _stream(stream))
+
+
+def dispatch_lu_cm(A, n: int, lda: int, AB, ldab: int, ipiv, d_info, stream=None) -> tuple[int, int, int]:
+    """dispatch_lu for a column-major A.  Returns (status, kl, ku)."""
+    kl, ku = ctypes.c_int(-1), ctypes.c_int(-1)
+    rc = load().dispatch_lu_cm(_ptr(A), n, lda, _ptr(AB), ldab, _ptr(ipiv), ctypes.addressof(kl),
+                               ctypes.addressof(ku), _ptr(d_info), _stream(stream))
     return rc, kl.value, ku.value
 
 

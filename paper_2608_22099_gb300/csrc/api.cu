@@ -37,6 +37,29 @@ int dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, doubl
   return bandlu::launch_dense_to_band(A, lda, n, kl, ku, AB, ldab, stream);
 }
 
+int detect_bandwidth_cm(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t stream) {
+  if (bad_n(n)) return -2;
+  if (A == nullptr && n > 0) return -1;
+  if (lda < max1(n)) return -3;
+  if (d_kl == nullptr) return -4;
+  if (d_ku == nullptr) return -5;
+  // read as row-major, the column-major A is its transpose: the lower and upper
+  // bandwidths trade places
+  return bandlu::launch_detect(A, n, lda, d_ku, d_kl, stream);
+}
+
+int dense_to_band_cm(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                     cudaStream_t stream) {
+  if (bad_n(n)) return -3;
+  if (A == nullptr && n > 0) return -1;
+  if (lda < max1(n)) return -2;
+  if (kl < 0) return -4;
+  if (ku < 0) return -5;
+  if (AB == nullptr && n > 0) return -6;
+  if (ldab < 2 * (int64_t)kl + ku + 1) return -7;
+  return bandlu::launch_dense_to_band_cm(A, lda, n, kl, ku, AB, ldab, stream);
+}
+
 int gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t stream) {
   if (bad_n(n)) return -1;
   if (kl < 0) return -2;
@@ -73,6 +96,35 @@ int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t lda
   *h_ku = h[1];
   if (!bandlu::predicate_banded(n, h[0], h[1], ldab)) return BANDLU_NOT_BANDED;
   rc = bandlu::launch_dense_to_band(A, lda, n, h[0], h[1], AB, ldab, stream);
+  if (rc != BANDLU_OK) return rc;
+  return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream);
+}
+
+int dispatch_lu_cm(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *h_kl,
+                   int *h_ku, int *d_info, cudaStream_t stream) {
+  if (A == nullptr && n > 0) return -1;
+  if (bad_n(n)) return -2;
+  if (lda < max1(n)) return -3;
+  if (AB == nullptr && n > 0) return -4;
+  if (ldab < 1) return -5;
+  if (ipiv == nullptr && n > 0) return -6;
+  if (h_kl == nullptr) return -7;
+  if (h_ku == nullptr) return -8;
+  if (d_info == nullptr) return -9;
+  int *d_klku = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&d_klku), 2 * sizeof(int), stream) != cudaSuccess)
+    return BANDLU_ERR_CUDA;
+  int rc = bandlu::launch_detect(A, n, lda, d_klku + 1, d_klku, stream);  // transposed view: (ku, kl)
+  int h[2] = {0, 0};
+  if (rc == BANDLU_OK && cudaMemcpyAsync(h, d_klku, sizeof(h), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    rc = BANDLU_ERR_CUDA;
+  if (cudaFreeAsync(d_klku, stream) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (cudaStreamSynchronize(stream) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  if (rc != BANDLU_OK) return rc;
+  *h_kl = h[0];
+  *h_ku = h[1];
+  if (!bandlu::predicate_banded(n, h[0], h[1], ldab)) return BANDLU_NOT_BANDED;
+  rc = bandlu::launch_dense_to_band_cm(A, lda, n, h[0], h[1], AB, ldab, stream);
   if (rc != BANDLU_OK) return rc;
   return bandlu::launch_gbtrf(n, h[0], h[1], AB, ldab, ipiv, d_info, stream);
 }

@@ -110,6 +110,9 @@ namespace bandlu {
 int launch_detect(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t s);
 int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
                          cudaStream_t s);
+// Column-major input, A(i,j) = A[i + j*lda].
+int launch_dense_to_band_cm(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                            cudaStream_t s);
 // allow_alloc = false keeps the launch free of device allocations (wide bands
 // then take the single-CTA kernel instead of the multi-CTA one, whose
 // hand-off flags live in stream-ordered scratch).

@@ -109,6 +109,24 @@ __global__ void __launch_bounds__(256) k_decide_convert_direct(const double *__r
   }
 }
 
+// Column-major input, A(i,j) = A[i + j*lda]: one thread per AB entry; AB
+// column j is A's column j shifted by kv - j, so consecutive threads read and
+// write consecutive addresses.
+__global__ void __launch_bounds__(256) k_dense_to_band_cm(const double *__restrict__ A, long long lda, long long n,
+                                                          int kl, int ku, double *__restrict__ AB, long long ldab) {
+  const long long kv = (long long)kl + ku;
+  const long long total = n * ldab;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long j = e / ldab;
+    const long long r = e - j * ldab;
+    const long long i = j - kv + r;
+    double v = 0.0;
+    if (r >= kl && r <= kv + kl && i >= 0 && i < n) v = A[i + j * lda];
+    AB[e] = v;
+  }
+}
+
 constexpr int kTileSmemMax = 96 * 1024;
 
 // Columns per tile for band storage of height ldab: enough blocks to cover the
@@ -165,6 +183,16 @@ int launch_decide_convert(const double *A, int64_t lda, int64_t n, int64_t ldab,
     if (blocks < 1) blocks = 1;
     k_decide_convert_direct<<<(unsigned)blocks, 256, 0, s>>>(A, lda, n, d_kl, d_ku, d_status, AB, ldab);
   }
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+int launch_dense_to_band_cm(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
+                            cudaStream_t s) {
+  if (n == 0) return BANDLU_OK;
+  long long blocks = (n * ldab + 255) / 256;
+  if (blocks > 152ll * 64) blocks = 152ll * 64;
+  k_dense_to_band_cm<<<(unsigned)blocks, 256, 0, s>>>(A, lda, n, kl, ku, AB, ldab);
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;
 }

@@ -215,3 +215,30 @@ def test_classify_matches_the_oracle(oracle_mod):
 ])
 def test_dispatch_lu_async_argument_checks(args, expect):
     assert bandlu.dispatch_lu_async(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((DEV, -1, 1, DEV, DEV), -2), ((0, 4, 4, DEV, DEV), -1), ((DEV, 4, 3, DEV, DEV), -3),
+    ((DEV, 4, 4, 0, DEV), -4), ((DEV, 4, 4, DEV, 0), -5),
+])
+def test_detect_bandwidth_cm_argument_checks(args, expect):
+    assert bandlu.detect_bandwidth_cm(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, 1, 1, DEV, 4), -1), ((DEV, 3, 4, 1, 1, DEV, 4), -2), ((DEV, 4, -1, 1, 1, DEV, 4), -3),
+    ((DEV, 4, 4, -1, 1, DEV, 4), -4), ((DEV, 4, 4, 1, -1, DEV, 4), -5), ((DEV, 4, 4, 1, 1, 0, 4), -6),
+    ((DEV, 4, 4, 1, 1, DEV, 3), -7),
+])
+def test_dense_to_band_cm_argument_checks(args, expect):
+    assert bandlu.dense_to_band_cm(*args, stream=0) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, 4, 4, DEV, 4, DEV, DEV), -1), ((DEV, -2, 4, DEV, 4, DEV, DEV), -2), ((DEV, 4, 2, DEV, 4, DEV, DEV), -3),
+    ((DEV, 4, 4, 0, 4, DEV, DEV), -4), ((DEV, 4, 4, DEV, 0, DEV, DEV), -5), ((DEV, 4, 4, DEV, 4, 0, DEV), -6),
+    ((DEV, 4, 4, DEV, 4, DEV, 0), -9),
+])
+def test_dispatch_lu_cm_argument_checks(args, expect):
+    rc, _, _ = bandlu.dispatch_lu_cm(*args, stream=0)
+    assert rc == expect
