@@ -298,6 +298,26 @@ def run_ours(args):
     ms_per_step = multirank.max_over_ranks(sum(step_ms), device=dev) / args.steps
     value = multirank.job_throughput(multirank.sum_over_ranks(flops, device=dev), ms_per_step * 1e-3) / 1e9
 
+    # the same step with the dispatch decision on the device (dispatch_lu_async: no host round trip)
+    sc = torch.zeros(4, dtype=torch.int32, device=dev)
+
+    def step_async():
+        bandlu.check(bandlu.dispatch_lu_async(A, n, n, AB, ldab, ipiv, sc[0:1], sc[1:2], sc[2:3], sc[3:4], stream),
+                     "dispatch_lu_async")
+    for _ in range(3):
+        step_async()
+    areps = min(args.steps, 50)
+    aev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(areps)]
+    for r in range(areps):
+        flush(r)
+        aev[r][0].record(stream)
+        step_async()
+        aev[r][1].record(stream)
+    torch.cuda.synchronize()
+    async_ms = statistics.mean(a.elapsed_time(b) for a, b in aev)
+    if tuple(int(v) for v in sc[:3].cpu()) != (kl, ku, 0):
+        raise RuntimeError("dispatch_lu_async disagrees with dispatch_lu")
+
     # stage breakdown through the same C ABI, CUDA events on the launching stream
     klku = torch.zeros(2, dtype=torch.int32, device=dev)
     AB2 = torch.zeros_like(AB)
@@ -402,7 +422,7 @@ def run_ours(args):
             "config": {"workload": WORKLOAD, "n": n, "kl": kl, "ku": ku, "ldab": ldab, "dist": "uniform[-1,1]",
                        "l2": "flushed between steps (512 MiB write, then a 256 MiB read that writes its dirty lines back)",
                        "parallelism": "replicas" if world > 1 else "single"},
-            "dispatch_ms": ms_per_step, "dense_lu_ms": dense_t,
+            "dispatch_ms": ms_per_step, "dispatch_async_ms": async_ms, "dense_lu_ms": dense_t,
             "speedup_over_dense": (dense_t / ms_per_step) if dense_t else None,
             "flops_per_step": flops, "stages": stages, "roofline": roofline,
             "cpu_baseline": cpu_baseline,
@@ -491,23 +511,25 @@ def run_workload_report(args):
         t_disp = timed(disp, reps)
         t_det = timed(det, reps)
         # the same dispatch with the decision on the device (no host round trip), and that call
-        # captured once in a CUDA graph and replayed
-        sc = torch.zeros(4, dtype=torch.int32, device=dev)
+        # captured once in a CUDA graph and replayed; for the bands its one-CTA kernels cover
+        # (wider bands take its block-wide fallback, seconds at n = 32768)
+        if kl <= 27 and 2 * kl + ku + 1 <= 256:
+            sc = torch.zeros(4, dtype=torch.int32, device=dev)
 
-        def dasync(st):
-            bandlu.check(bandlu.dispatch_lu_async(A, n, n, AB, ldab, ipiv, sc[0:1], sc[1:2], sc[2:3], sc[3:4], st),
-                         "dispatch_lu_async")
-        for _ in range(3):
-            dasync(stream)
-        t_async = timed(lambda: dasync(stream), reps)
-        gs = torch.cuda.Stream()
-        torch.cuda.synchronize()
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph, stream=gs):
-            dasync(gs)
-        graph.replay()
-        t_graph = timed(graph.replay, reps)
-        out.update({"dispatch_async_ms": t_async * 1e3, "dispatch_graph_ms": t_graph * 1e3})
+            def dasync(st):
+                bandlu.check(bandlu.dispatch_lu_async(A, n, n, AB, ldab, ipiv, sc[0:1], sc[1:2], sc[2:3], sc[3:4],
+                                                      st), "dispatch_lu_async")
+            for _ in range(3):
+                dasync(stream)
+            t_async = timed(lambda: dasync(stream), reps)
+            gs = torch.cuda.Stream()
+            torch.cuda.synchronize()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=gs):
+                dasync(gs)
+            graph.replay()
+            t_graph = timed(graph.replay, reps)
+            out.update({"dispatch_async_ms": t_async * 1e3, "dispatch_graph_ms": t_graph * 1e3})
         rc, dkl, dku = res["rc"]
         out.update({"status": rc, "detected_kl": dkl, "detected_ku": dku, "dispatch_ms": t_disp * 1e3,
                     "detect_us": t_det * 1e6, "detect_gbs": 8.0 * n * n / t_det / 1e9,
@@ -533,6 +555,18 @@ def run_workload_report(args):
                 xb.copy_(b0)
                 bandlu.check(bandlu.gbtrs(n, kl, ku, 1, AB2, ldab, ipiv, xb, n, stream), "gbtrs")
             t_sol = timed(sol, max(1, min(reps, 5)))
+            if n <= 20000:
+                # the lower-triangular branch of the backslash dispatch on the matrix's own lower
+                # triangle (bandwidth kl, read in place from the dense matrix)
+                Lm = torch.tril(A)
+                info2 = torch.zeros(1, dtype=torch.int32, device=dev)
+
+                def trs():
+                    xb.copy_(b0)
+                    bandlu.check(bandlu.trsv_band(1, n, kl, Lm, n, xb, n, 1, info2, stream), "trsv_band")
+                trs()
+                out["trsv_lower_1rhs_ms"] = timed(trs, max(1, min(reps, 5))) * 1e3
+                del Lm
             out.update({"convert_us": t_conv * 1e6, "gbtrf_ms": t_fac * 1e3, "gbtrf_gflops": flops / t_fac / 1e9,
                         "gbtrf_ns_per_column": t_fac / n * 1e9, "flops": flops,
                         "gflops_dispatch": flops / t_disp / 1e9, "gbtrs_1rhs_ms": t_sol * 1e3,
