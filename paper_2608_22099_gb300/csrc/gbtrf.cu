@@ -126,6 +126,16 @@ struct WinShared {
 };
 
 
+// Asynchronous global -> shared copies (the I/O warp's row prefetch).
+__device__ __forceinline__ void cp_async8(double *dst, const double *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"((unsigned)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// every group but the newest has completed
+__device__ __forceinline__ void cp_async_wait_prior() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // Out of line, so that the rarely taken division is not if-converted into the
 // pivot chain of the panel warp.
 __device__ __noinline__ double div_slow(double x) { return 1.0 / x; }
@@ -251,14 +261,14 @@ __device__ __forceinline__ void window_factor(int n, int kl, int ku, double *__r
     // ---------------- I/O warp ----------------
     // Step j's pivot, U diagonal, U(j, j+1), U(j, j+2) and multipliers go to
     // global memory; then the row prefetch: row j-1+R enters the slot that row
-    // j-1 left; it is fetched in step j and stored in step j+1 (a whole step for
-    // the global loads to land).
+    // j-1 left, copied straight into it with cp.async.  The copy issued in step
+    // j is waited for at the end of step j+1, before this warp's arrival at
+    // kBarPub(j+2): the row is first read in step j+3 (the panel's column j+4,
+    // after kBarCol(j+2), which the helper reaches after kBarPub(j+2)), and the
+    // load has two steps to land instead of stalling every step on it.
     int pfo[PF];
 #pragma unroll
     for (int k = 0; k < PF; ++k) pfo[k] = (kDelta + lane + 32 * k) % CS;
-    double pf[PF];
-    bool have_pf = false;
-    int pf_rb = 0, pf_q = 0;
     int qj = 0;
     unsigned ph_pub = 0;
     for (int j = 0; j < n; ++j) {
@@ -273,38 +283,37 @@ __device__ __forceinline__ void window_factor(int n, int kl, int ku, double *__r
         if (kv >= 1 && j + 1 < n) AB[(kv - 1) + (long long)(j + 1) * ldab] = sh.meta[b].u1;
       }
       if (lane >= 1 && lane <= km) AB[(kv + lane) + (long long)j * ldab] = sh.pk[b][lane].l;
-      if (have_pf) {
-#pragma unroll
-        for (int k = 0; k < PF; ++k) {
-          if (lane + 32 * k < CS) {
-            int q = pf_q + pfo[k];
-            if (q >= CS) q -= CS;
-            W[pf_rb + q] = pf[k];
-          }
-        }
-        have_pf = false;
-      }
       if (j >= 1 && j - 1 + R < n) {
         const int i = j - 1 + R;
-        pf_rb = sh.pk[b][R - 1].rb;
-        pf_q = qj;
-        have_pf = true;
+        const int rb = sh.pk[b][R - 1].rb;
 #pragma unroll
         for (int k = 0; k < PF; ++k) {
           const int kk = lane + 32 * k;
-          const int c = i - kl + kk;
-          pf[k] = (kk < CS && c <= i + ku && c < n) ? AB[(kv + i - c) + (long long)c * ldab] : 0.0;
+          if (kk < CS) {
+            int q = qj + pfo[k];
+            if (q >= CS) q -= CS;
+            const int c = i - kl + kk;  // >= 0
+            if (c <= i + ku && c < n)
+              cp_async8(W + rb + q, AB + (kv + i - c) + (long long)c * ldab);
+            else
+              W[rb + q] = 0.0;
+          }
         }
       }
+      cp_async_commit();
+      cp_async_wait_prior();  // the copy of step j-1 has landed
       qj = (qj + 1 == CS) ? 0 : qj + 1;
     }
+    cp_async_wait_all();
   } else if ((warp & 3) != 0) {
     // ---------------- updater warps: columns j+3 .. j+kv ----------------
     // Updater index of this warp.  The order puts the warps that also take the
     // last, partial round of elements on different SMSPs, so that the FP64
     // instructions of a step spread evenly over the SMSPs' pipes.
-    constexpr int kUw[16] = {-1, 0, 2, 3, -1, 1, 4, 5, -1, 6, 7, 8, -1, -1, 9, 10};
-    const int uw = kUw[warp];  // 0..kNU-1
+    // warp -> updater index {-, 0, 2, 3, -, 1, 4, 5, -, 6, 7, 8, -, -, 9, 10}, four bits
+    // per warp in one constant (a table would be a local-memory array)
+    constexpr unsigned long long kUwPacked = 0xA9FF876F541F320Full;
+    const int uw = (int)((kUwPacked >> (4 * warp)) & 15ull);  // 0..kNU-1
     const int tid_u = uw * 32 + lane;
     const int ncols = kv > 2 ? kv - 2 : 0;
     const int E = ncols * (kl + 1);
