@@ -57,10 +57,17 @@ __device__ __forceinline__ int warp_argmax_first(unsigned long long key) {
   return __ffs(win) - 1;
 }
 
-// As warp_argmax_first, and *all_zero tells whether every key is zero.
+// As warp_argmax_first, and *all_zero tells whether every key is zero.  When
+// one lane alone holds the largest high word (the usual case) it is the
+// winner and the reduction over the low words is skipped.
 __device__ __forceinline__ int warp_argmax_first_z(unsigned long long key, bool *all_zero) {
   const unsigned hi = (unsigned)(key >> 32), lo = (unsigned)key;
   const unsigned mhi = __reduce_max_sync(FULL, hi);
+  const unsigned top = __ballot_sync(FULL, hi == mhi);
+  if (__popc(top) == 1) {  // uniform; then mhi > 0 (mhi == 0 would put every lane in top)
+    *all_zero = false;
+    return __ffs(top) - 1;
+  }
   const unsigned lo2 = (hi == mhi) ? lo : 0u;
   const unsigned mlo = __reduce_max_sync(FULL, lo2);
   const unsigned win = __ballot_sync(FULL, hi == mhi && lo == mlo);

@@ -14,10 +14,14 @@
 //    owns the critical path: it keeps the pivot column in registers (lane t =
 //    row j+t), finds the pivot with an exact integer argmax, forms the
 //    multipliers, and itself applies step j to column j+1 so that step j+1
-//    can start at once.  Warps 1..3 (updaters) apply step j to columns
-//    j+2..j+kv (column j+2 first, which the panel needs next), stream the
-//    finished U row to global memory and prefetch the rows that enter the
-//    window.  Hand-offs are two named barriers per step (see kBarPub/kBarCol).
+//    can start at once.  The helper warp applies step j to column j+2 (which
+//    the panel needs next), 11 updater warps (none on the panel's SMSP) to
+//    columns j+3..j+kv and write the finished U row, and the I/O warp writes
+//    the pivot and multipliers and copies the rows that enter the window into
+//    their slots (cp.async).  Hand-offs are two named barriers per step (see
+//    kBarPub/kBarCol).  (Two more updater warps on the panel's SMSP were
+//    measured: faster for kl = 27, slower for kl <= 16, where the panel's
+//    FP64 instructions then queue behind theirs.)
 //
 //  * k_gbtrf_generic (any kl, ku).  One CTA works directly on AB in global
 //    memory (the active window stays L2-resident), one column at a time.

@@ -10,6 +10,18 @@
 namespace bandlu {
 namespace regwin {
 
+// warp_argmax_first_z without its shortcut: both reductions, always.  Several
+// segments' argmaxes in a row (S > 1) run faster without the shortcut's branch.
+__device__ __forceinline__ int argmax_two_pass(unsigned long long key, bool *all_zero) {
+  const unsigned hi = (unsigned)(key >> 32), lo = (unsigned)key;
+  const unsigned mhi = __reduce_max_sync(FULL, hi);
+  const unsigned lo2 = (hi == mhi) ? lo : 0u;
+  const unsigned mlo = __reduce_max_sync(FULL, lo2);
+  const unsigned win = __ballot_sync(FULL, hi == mhi && lo == mlo);
+  *all_zero = (mhi | mlo) == 0u;
+  return __ffs(win) - 1;
+}
+
 constexpr int kWinPrefetch = 8;  // entering rows a window keeps in flight
 
 // Banded elimination with the active window in registers, in place on band
@@ -89,7 +101,7 @@ __device__ __forceinline__ void window_gbtrf(double *const (&abs)[S], int ldab, 
 #pragma unroll
       for (int t = 0; t < S; ++t) {
         bool allz;
-        const int wt = warp_argmax_first_z(seg == t ? key : 0ull, &allz);
+        const int wt = S == 1 ? warp_argmax_first_z(key, &allz) : argmax_two_pass(seg == t ? key : 0ull, &allz);
         if (seg == t) {
           win = wt;
           zp = allz;
