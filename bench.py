@@ -361,7 +361,9 @@ def run_ours(args):
                     "frac": achieved / FP64_PEAK_GFLOPS, "traffic": profiled_traffic("k_gbtrf_window"),
                     "kernel": "k_gbtrf_window",
                     "peak_source": "nominal FP64 (152 SMs x 2 DFMA/clk x 2 flop x 2.07 GHz)",
-                    "note": "one matrix is one serial pivot chain on one SM: latency-bound, see ns_per_column"}
+                    "frac_of_one_sm": achieved / (FP64_PEAK_GFLOPS / 152),
+                    "note": "one matrix is one serial pivot chain on one SM (one CTA): latency-bound, see "
+                            "ns_per_column; frac_of_one_sm is against that SM's share of the peak"}
     elif dominant == "detect":
         roofline = {"bound": "hbm", "achieved": detect_bytes / t_detect / 1e9, "peak": hbm_peak, "unit": "GB/s",
                     "frac": detect_bytes / t_detect / 1e9 / hbm_peak, "traffic": profiled_traffic("k_detect_vec"),

@@ -35,10 +35,17 @@ namespace trwin {
 
 // Coefficients of the sweeps.  k is the step; t >= 0 the offset from the
 // eliminated position.
+// at(k, t): the coefficient's address.  prefetch(k, kw, n, lane): called once
+// per step k by every lane, asks L2 for data the sweep reads kPrefetchSteps
+// steps later (a no-op for the band storage, which the factorisation has just
+// left in L2).
+constexpr int kPrefetchSteps = 48;
+
 struct GbLower {  // forward half of xGBTRS: multipliers l_{k+t,k} = AB(kv+t, k)
   const double *AB;
   int ldab, kv;
   __device__ __forceinline__ const double *at(int k, int t) const { return AB + (kv + t) + (long long)k * ldab; }
+  __device__ __forceinline__ void prefetch(int, int, int, int) const {}
 };
 struct GbUpper {  // backward half of xGBTRS: j = n-1-k, U(j-t, j) = AB(kv-t, j)
   const double *AB;
@@ -46,11 +53,25 @@ struct GbUpper {  // backward half of xGBTRS: j = n-1-k, U(j-t, j) = AB(kv-t, j)
   __device__ __forceinline__ const double *at(int k, int t) const {
     return AB + (kv - t) + (long long)(n - 1 - k) * ldab;
   }
+  __device__ __forceinline__ void prefetch(int, int, int, int) const {}
 };
+// In the dense matrix the coefficients of one step lie in different rows (one
+// 32-byte sector each), but row m's band segment -- used over kw consecutive
+// steps -- is contiguous: lane L prefetches the L-th 128-byte line of the
+// segment of the row whose first use is kPrefetchSteps steps ahead.
+__device__ __forceinline__ void prefetch_l2_line(const double *p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
 struct DenseLower {  // lower triangular, row-major dense: L(k+t, k) = A[(k+t)*lda + k]
   const double *A;
   long long lda;
   __device__ __forceinline__ const double *at(int k, int t) const { return A + (long long)(k + t) * lda + k; }
+  // row m = k + kw + kPrefetchSteps is first read at step m - kw; its segment is
+  // A[m*lda + m-kw .. m-1]
+  __device__ __forceinline__ void prefetch(int k, int kw, int n, int lane) const {
+    const int m = k + kw + kPrefetchSteps;
+    if (m < n && lane * 16 < kw) prefetch_l2_line(A + (long long)m * lda + (m - kw) + lane * 16);
+  }
 };
 struct DenseUpper {  // upper triangular, row-major dense: j = n-1-k, U(j-t, j) = A[(j-t)*lda + j]
   const double *A;
@@ -59,6 +80,12 @@ struct DenseUpper {  // upper triangular, row-major dense: j = n-1-k, U(j-t, j) 
   __device__ __forceinline__ const double *at(int k, int t) const {
     const int j = n - 1 - k;
     return A + (long long)(j - t) * lda + j;
+  }
+  // row m = j - kw - kPrefetchSteps is first read at column m + kw; its segment
+  // is A[m*lda + m+1 .. m+kw]
+  __device__ __forceinline__ void prefetch(int k, int kw, int, int lane) const {
+    const int m = n - 1 - k - kw - kPrefetchSteps;
+    if (m >= 0 && lane * 16 < kw) prefetch_l2_line(A + (long long)m * lda + (m + 1) + lane * 16);
   }
 };
 
@@ -188,6 +215,7 @@ __device__ __forceinline__ void sweep(double *b, int n, int kw, const Src &src, 
       if (lane == (k & 31)) b[row(k)] = x;
       put(w, k, en[s], lane);  // position k leaves, position k+W enters
       fill(s, k + kPf);
+      src.prefetch(k, kw, n, lane);
     }
   }
 }
