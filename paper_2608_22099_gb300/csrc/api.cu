@@ -2,8 +2,27 @@
 // launches of detect.cu, convert.cu, gbtrf.cu, gbtrf_wide.cu, gbtrs.cu,
 // trsolve.cu and batched.cu.
 #include <climits>
+#include <mutex>
+#include <set>
+#include <utility>
 
 #include "common.cuh"
+
+namespace bandlu {
+
+bool allow_dynamic_smem(const void *kernel, int bytes) {
+  static std::mutex mu;
+  static std::set<std::pair<const void *, int>> done;  // (kernel, device) pairs already opted in
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  std::lock_guard<std::mutex> lock(mu);
+  if (done.count({kernel, dev})) return true;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess) return false;
+  done.insert({kernel, dev});
+  return true;
+}
+
+}  // namespace bandlu
 
 namespace {
 

@@ -148,13 +148,7 @@ int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku
   const int T = tile_columns(n, ldab);
   if (T > 0) {
     const size_t smem = (size_t)T * per_col;
-    static bool attr_set = false;
-    if (!attr_set) {
-      if (cudaFuncSetAttribute(k_dense_to_band_tiled, cudaFuncAttributeMaxDynamicSharedMemorySize, kTileSmemMax) !=
-          cudaSuccess)
-        return BANDLU_ERR_CUDA;
-      attr_set = true;
-    }
+    if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_dense_to_band_tiled), kTileSmemMax)) return BANDLU_ERR_CUDA;
     const long long blocks = (n + T - 1) / T;
     k_dense_to_band_tiled<<<(unsigned)blocks, 256, smem, s>>>(A, lda, n, kl, ku, AB, ldab, T);
   } else {
@@ -172,9 +166,8 @@ int launch_decide_convert(const double *A, int64_t lda, int64_t n, int64_t ldab,
   const int T = n > 0 ? tile_columns(n, ldab) : 0;  // n == 0: the direct kernel records the decision
   if (T > 0) {
     const size_t smem = (size_t)T * ldab * sizeof(double);
-    static const bool attr = cudaFuncSetAttribute(k_decide_convert_tiled, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                  kTileSmemMax) == cudaSuccess;
-    if (!attr) return BANDLU_ERR_CUDA;
+    if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_decide_convert_tiled), kTileSmemMax))
+      return BANDLU_ERR_CUDA;
     k_decide_convert_tiled<<<(unsigned)((n + T - 1) / T), 256, smem, s>>>(A, lda, n, d_kl, d_ku, d_status, AB, ldab,
                                                                           T);
   } else {

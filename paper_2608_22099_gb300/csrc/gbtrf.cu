@@ -567,13 +567,7 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_on_device(int n, doubl
 template <int K, int PF>
 int launch_window(long long n, int kl, int ku, double *AB, long long ldab, int *ipiv, int *d_info, size_t smem,
                   cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(k_gbtrf_window<K, PF>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
-        cudaSuccess)
-      return BANDLU_ERR_CUDA;
-    attr = true;
-  }
+  if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_window<K, PF>), 200 * 1024)) return BANDLU_ERR_CUDA;
   k_gbtrf_window<K, PF><<<1, kWarps * 32, smem, s>>>((int)n, kl, ku, AB, ldab, ipiv, d_info);
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;
@@ -631,10 +625,7 @@ int launch_gbtrf_on_device(int64_t n, double *AB, int64_t ldab, int *ipiv, const
   // CS = 2*kl+ku+1 <= min(ldab, 256) column slots of R = kl+1+kDelta rows
   const long long cs = ldab < 256 ? ldab : 256;
   const size_t smem = (size_t)((kWinMaxKl + 1 + kDelta) * cs) * sizeof(double);
-  static const bool attr =
-      cudaFuncSetAttribute(k_gbtrf_on_device, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) ==
-      cudaSuccess;
-  if (!attr) return BANDLU_ERR_CUDA;
+  if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_on_device), 200 * 1024)) return BANDLU_ERR_CUDA;
   k_gbtrf_on_device<<<1, kWarps * 32, smem, s>>>((int)n, AB, ldab, ipiv, d_kl, d_ku, d_status, d_info, smem);
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;

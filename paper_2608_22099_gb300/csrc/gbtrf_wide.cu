@@ -685,13 +685,7 @@ __global__ void __launch_bounds__(Lay<CW>::kThreads, 1)
 template <int CW, int RPT>
 int launch_rpt(const Geo &g, int grid, size_t smem, double *AB, int *ipiv, int *d_info, int *flags, cudaStream_t s) {
   constexpr int kThreads = Lay<CW>::kThreads;
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(k_gbtrf_wide<CW, RPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
-        cudaSuccess)
-      return BANDLU_ERR_CUDA;
-    attr = true;
-  }
+  if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_wide<CW, RPT>), 200 * 1024)) return BANDLU_ERR_CUDA;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_gbtrf_wide<CW, RPT>, kThreads, smem) != cudaSuccess)
     return BANDLU_ERR_CUDA;

@@ -216,12 +216,7 @@ int launch_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int6
   int WS = 1;
   while (WS < win + 32) WS <<= 1;
   if (n <= INT_MAX / 2 && nrhs <= INT_MAX && (size_t)WS * sizeof(double) <= 96 * 1024) {
-    static bool attr = false;
-    if (!attr) {
-      if (cudaFuncSetAttribute(k_gbtrs_cta, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024) != cudaSuccess)
-        return BANDLU_ERR_CUDA;
-      attr = true;
-    }
+    if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrs_cta), 96 * 1024)) return BANDLU_ERR_CUDA;
     k_gbtrs_cta<<<(unsigned)nrhs, 256, (size_t)WS * sizeof(double), s>>>((int)n, kl, ku, WS, AB, ldab, ipiv, B, ldb,
                                                                         d_info);
     BANDLU_CHECK_LAUNCH();
