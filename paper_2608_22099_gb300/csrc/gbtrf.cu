@@ -191,7 +191,9 @@ __device__ __forceinline__ void window_factor(int n, int kl, int ku, double *__r
       bool myspec;
       const double myr = rcp_rn_fast(cur, &myspec);  // integer pipes
       bool zp;  // exact zero pivot (then p == 0)
-      const int p = warp_argmax_first_z(valid ? pivot_abs_key(cur, lane == 0) : 0ull, &zp);
+      // (the two-pass form: here the shortcut's branch costs the panel more than
+      // the second reduction it saves)
+      const int p = regwin::argmax_two_pass(valid ? pivot_abs_key(cur, lane == 0) : 0ull, &zp);
       // interchange rows j and j+p: lanes 0 and p trade their values and slots
       const int src = lane == 0 ? p : (lane == p ? 0 : lane);
       slot_reg = __shfl_sync(FULL, slot_reg, src);
