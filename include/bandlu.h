@@ -25,7 +25,9 @@
  *    invalid (nothing is enqueued), or one of the positive codes below.  No
  *    entry point traps, asserts or hangs on the device.
  *  - Indexing is 64-bit throughout; n is limited to 2^31 - 1 and kl, ku to
- *    n - 1 (they are int32 in the outputs).
+ *    n - 1 (they are int32 in the outputs).  A leading dimension or stride
+ *    whose extent over the matrix (or batch) does not fit a 64-bit offset is
+ *    rejected like any other invalid argument.
  */
 #ifndef BANDLU_H
 #define BANDLU_H

@@ -28,6 +28,15 @@ namespace {
 
 inline bool bad_n(int64_t n) { return n < 0 || n > (int64_t)INT_MAX; }
 inline int64_t max1(int64_t n) { return n > 1 ? n : 1; }
+// a leading dimension whose n columns' (or rows') extent n * ld would not fit
+// the 64-bit offsets the kernels compute
+inline bool bad_ld(int64_t n, int64_t ld) { return ld < max1(n) || ld > INT64_MAX / max1(n); }
+// an extent ld per item that would overflow 64-bit offsets over count items
+inline bool too_long(int64_t count, int64_t ld) { return ld > INT64_MAX / max1(count); }
+// the same for strides between the matrices of a batch
+inline bool bad_stride(int64_t count, int64_t stride, int64_t minimum) {
+  return stride < minimum || (count > 0 && stride > INT64_MAX / count);
+}
 
 }  // namespace
 
@@ -38,7 +47,7 @@ const char *bandlu_version(void) { return "bandlu 0.1 (sm_103a)"; }
 int detect_bandwidth(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t stream) {
   if (bad_n(n)) return -2;
   if (A == nullptr && n > 0) return -1;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (d_kl == nullptr) return -4;
   if (d_ku == nullptr) return -5;
   return bandlu::launch_detect(A, n, lda, d_kl, d_ku, stream);
@@ -48,18 +57,18 @@ int dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, doubl
                   cudaStream_t stream) {
   if (bad_n(n)) return -3;
   if (A == nullptr && n > 0) return -1;
-  if (lda < max1(n)) return -2;
+  if (bad_ld(n, lda)) return -2;
   if (kl < 0) return -4;
   if (ku < 0) return -5;
   if (AB == nullptr && n > 0) return -6;
-  if (ldab < 2 * (int64_t)kl + ku + 1) return -7;
+  if (ldab < 2 * (int64_t)kl + ku + 1 || too_long(n, ldab)) return -7;
   return bandlu::launch_dense_to_band(A, lda, n, kl, ku, AB, ldab, stream);
 }
 
 int detect_bandwidth_cm(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t stream) {
   if (bad_n(n)) return -2;
   if (A == nullptr && n > 0) return -1;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (d_kl == nullptr) return -4;
   if (d_ku == nullptr) return -5;
   // read as row-major, the column-major A is its transpose: the lower and upper
@@ -71,11 +80,11 @@ int dense_to_band_cm(const double *A, int64_t lda, int64_t n, int kl, int ku, do
                      cudaStream_t stream) {
   if (bad_n(n)) return -3;
   if (A == nullptr && n > 0) return -1;
-  if (lda < max1(n)) return -2;
+  if (bad_ld(n, lda)) return -2;
   if (kl < 0) return -4;
   if (ku < 0) return -5;
   if (AB == nullptr && n > 0) return -6;
-  if (ldab < 2 * (int64_t)kl + ku + 1) return -7;
+  if (ldab < 2 * (int64_t)kl + ku + 1 || too_long(n, ldab)) return -7;
   return bandlu::launch_dense_to_band_cm(A, lda, n, kl, ku, AB, ldab, stream);
 }
 
@@ -84,7 +93,7 @@ int gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d
   if (kl < 0) return -2;
   if (ku < 0) return -3;
   if (AB == nullptr && n > 0) return -4;
-  if (ldab < 2 * (int64_t)kl + ku + 1) return -5;
+  if (ldab < 2 * (int64_t)kl + ku + 1 || too_long(n, ldab)) return -5;
   if (ipiv == nullptr && n > 0) return -6;
   if (d_info == nullptr) return -7;
   return bandlu::launch_gbtrf(n, kl, ku, AB, ldab, ipiv, d_info, stream);
@@ -94,9 +103,9 @@ int dispatch_lu(const double *A, int64_t n, int64_t lda, double *AB, int64_t lda
                 int *d_info, cudaStream_t stream) {
   if (A == nullptr && n > 0) return -1;
   if (bad_n(n)) return -2;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (AB == nullptr && n > 0) return -4;
-  if (ldab < 1) return -5;
+  if (ldab < 1 || too_long(n, ldab)) return -5;
   if (ipiv == nullptr && n > 0) return -6;
   if (h_kl == nullptr) return -7;
   if (h_ku == nullptr) return -8;
@@ -123,9 +132,9 @@ int dispatch_lu_cm(const double *A, int64_t n, int64_t lda, double *AB, int64_t 
                    int *h_ku, int *d_info, cudaStream_t stream) {
   if (A == nullptr && n > 0) return -1;
   if (bad_n(n)) return -2;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (AB == nullptr && n > 0) return -4;
-  if (ldab < 1) return -5;
+  if (ldab < 1 || too_long(n, ldab)) return -5;
   if (ipiv == nullptr && n > 0) return -6;
   if (h_kl == nullptr) return -7;
   if (h_ku == nullptr) return -8;
@@ -152,7 +161,7 @@ int dispatch_lu_async(const double *A, int64_t n, int64_t lda, double *AB, int64
                       int *d_ku, int *d_status, int *d_info, cudaStream_t stream) {
   if (A == nullptr && n > 0) return -1;
   if (bad_n(n)) return -2;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (AB == nullptr && n > 0) return -4;
   if (ldab < 1 || ldab > (int64_t)INT_MAX) return -5;
   if (ipiv == nullptr && n > 0) return -6;
@@ -174,10 +183,10 @@ int gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t lda
   if (ku < 0) return -3;
   if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -4;
   if (AB == nullptr && work) return -5;
-  if (ldab < 2 * (int64_t)kl + ku + 1) return -6;
+  if (ldab < 2 * (int64_t)kl + ku + 1 || too_long(n, ldab)) return -6;
   if (ipiv == nullptr && work) return -7;
   if (B == nullptr && work) return -8;
-  if (ldb < max1(n)) return -9;
+  if (ldb < max1(n) || too_long(nrhs, ldb)) return -9;
   return bandlu::launch_gbtrs(n, kl, ku, nrhs, AB, ldab, ipiv, B, ldb, nullptr, stream);
 }
 
@@ -186,12 +195,12 @@ int dispatch_solve(const double *A, int64_t n, int64_t lda, double *B, int64_t l
   const bool work = n > 0 && nrhs > 0;
   if (A == nullptr && n > 0) return -1;
   if (bad_n(n)) return -2;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (B == nullptr && work) return -4;
-  if (ldb < max1(n)) return -5;
+  if (ldb < max1(n) || too_long(nrhs, ldb)) return -5;
   if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -6;
   if (AB == nullptr && n > 0) return -7;
-  if (ldab < 1) return -8;
+  if (ldab < 1 || too_long(n, ldab)) return -8;
   if (ipiv == nullptr && n > 0) return -9;
   if (h_kl == nullptr) return -10;
   if (h_ku == nullptr) return -11;
@@ -209,9 +218,9 @@ int trsv_band(int lower, int64_t n, int k, const double *A, int64_t lda, double 
   if (bad_n(n)) return -2;
   if (k < 0 || (n > 0 && k > n - 1)) return -3;
   if (A == nullptr && n > 0) return -4;
-  if (lda < max1(n)) return -5;
+  if (bad_ld(n, lda)) return -5;
   if (B == nullptr && work) return -6;
-  if (ldb < max1(n)) return -7;
+  if (ldb < max1(n) || too_long(nrhs, ldb)) return -7;
   if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -8;
   if (d_info == nullptr) return -9;
   return bandlu::launch_trsv(lower == 1, n, k, A, lda, B, ldb, nrhs, d_info, stream);
@@ -222,9 +231,9 @@ int diag_solve(int64_t n, const double *A, int64_t lda, double *B, int64_t ldb, 
   const bool work = n > 0 && nrhs > 0;
   if (bad_n(n)) return -1;
   if (A == nullptr && n > 0) return -2;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (B == nullptr && work) return -4;
-  if (ldb < max1(n)) return -5;
+  if (ldb < max1(n) || too_long(nrhs, ldb)) return -5;
   if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -6;
   if (d_info == nullptr) return -7;
   return bandlu::launch_diag_solve(n, A, lda, B, ldb, nrhs, d_info, stream);
@@ -242,12 +251,12 @@ int dispatch_backslash(const double *A, int64_t n, int64_t lda, double *B, int64
   const bool work = n > 0 && nrhs > 0;
   if (A == nullptr && n > 0) return -1;
   if (bad_n(n)) return -2;
-  if (lda < max1(n)) return -3;
+  if (bad_ld(n, lda)) return -3;
   if (B == nullptr && work) return -4;
-  if (ldb < max1(n)) return -5;
+  if (ldb < max1(n) || too_long(nrhs, ldb)) return -5;
   if (nrhs < 0 || nrhs > (int64_t)INT_MAX) return -6;
   if (AB == nullptr && n > 0) return -7;
-  if (ldab < 1) return -8;
+  if (ldab < 1 || too_long(n, ldab)) return -8;
   if (ipiv == nullptr && n > 0) return -9;
   if (h_kl == nullptr) return -10;
   if (h_ku == nullptr) return -11;
@@ -291,14 +300,14 @@ int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA
   const bool work = n > 0 && batch > 0;
   if (A == nullptr && work) return -1;
   if (bad_n(n)) return -2;
-  if (lda < max1(n)) return -3;
-  if (strideA < n * lda) return -4;
+  if (bad_ld(n, lda)) return -3;
+  if (bad_stride(batch, strideA, n * lda)) return -4;
   if (batch < 0) return -5;
   if (AB == nullptr && work) return -6;
   if (ldab < 1 || ldab > (int64_t)INT_MAX) return -7;
-  if (strideAB < n * ldab) return -8;
+  if (bad_stride(batch, strideAB, n * ldab)) return -8;
   if (ipiv == nullptr && work) return -9;
-  if (strideP < n) return -10;
+  if (bad_stride(batch, strideP, n)) return -10;
   if ((d_kl == nullptr || d_ku == nullptr || d_info == nullptr || d_status == nullptr) && batch > 0) {
     if (d_kl == nullptr) return -11;
     if (d_ku == nullptr) return -12;

@@ -51,9 +51,10 @@ extern "C" int dispatch_lu_noalloc(const double *A, int64_t n, int64_t lda, doub
                                    int *h_kl, int *h_ku, int *d_info, cudaStream_t stream) {
   if (A == nullptr && n > 0) return -1;
   if (n < 0 || n > (int64_t)INT32_MAX) return -2;
-  if (lda < (n > 1 ? n : 1)) return -3;
+  const int64_t n1 = n > 1 ? n : 1;
+  if (lda < n1 || lda > INT64_MAX / n1) return -3;
   if (AB == nullptr && n > 0) return -4;
-  if (ldab < 1) return -5;
+  if (ldab < 1 || ldab > INT64_MAX / n1) return -5;
   if (ipiv == nullptr && n > 0) return -6;
   if (h_kl == nullptr) return -7;
   if (h_ku == nullptr) return -8;

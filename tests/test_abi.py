@@ -242,3 +242,23 @@ def test_dense_to_band_cm_argument_checks(args, expect):
 def test_dispatch_lu_cm_argument_checks(args, expect):
     rc, _, _ = bandlu.dispatch_lu_cm(*args, stream=0)
     assert rc == expect
+
+
+BIG = 1 << 62  # a leading dimension or stride whose extent over the matrix would overflow 64 bits
+
+
+@pytest.mark.parametrize("call,expect", [
+    (lambda: bandlu.detect_bandwidth(DEV, 4, BIG, DEV, DEV, stream=0), -3),
+    (lambda: bandlu.dense_to_band(DEV, BIG, 4, 1, 1, DEV, 4, stream=0), -2),
+    (lambda: bandlu.dense_to_band(DEV, 4, 4, 1, 1, DEV, BIG, stream=0), -7),
+    (lambda: bandlu.gbtrf(4, 1, 1, DEV, BIG, DEV, DEV, stream=0), -5),
+    (lambda: bandlu.gbtrs(4, 1, 1, 8, DEV, 4, DEV, DEV, BIG, stream=0), -9),
+    (lambda: bandlu.dispatch_lu(DEV, 4, BIG, DEV, 4, DEV, DEV, stream=0)[0], -3),
+    (lambda: bandlu.dispatch_lu_noalloc(DEV, 4, BIG, DEV, 4, DEV, DEV, stream=0)[0], -3),
+    (lambda: bandlu.dispatch_lu_noalloc(DEV, 4, 4, DEV, BIG, DEV, DEV, stream=0)[0], -5),
+    (lambda: bandlu.dispatch_lu_batched(DEV, 4, 4, BIG, 8, DEV, 4, 16, DEV, 4, DEV, DEV, DEV, DEV, stream=0), -4),
+    (lambda: bandlu.dispatch_lu_batched(DEV, 4, 4, 16, 8, DEV, 4, BIG, DEV, 4, DEV, DEV, DEV, DEV, stream=0), -8),
+    (lambda: bandlu.trsv_band(1, 4, 1, DEV, 4, DEV, BIG, 8, DEV, stream=0), -7),
+])
+def test_overflowing_extents_are_rejected(call, expect):
+    assert call() == expect
