@@ -6,10 +6,11 @@
 //  * k_first_zero_diag: the xTRTRS singularity check, info = first i with
 //    A(i,i) == 0 (1-based) or 0; the solves read it on the device and leave B
 //    as it is when it is nonzero.
-//  * k_trsv_lower / k_trsv_upper: one warp per right-hand side, a register
-//    window of the right-hand side (trwin.cuh) for k < 512: the column-oriented
-//    substitution of xTBSV with the reference BLAS's zero test and the IEEE
-//    quotient (div_known).
+//  * k_trsv_window<RW, kPf, kLower>: one warp per right-hand side, a register
+//    window of the right-hand side (trwin.cuh) for k + 1 <= 512: the
+//    column-oriented substitution of xTBSV with the reference BLAS's zero test
+//    and the IEEE quotient (div_known); each row's band segment is asked of L2
+//    ahead of its first use (trwin's DenseLower / DenseUpper sources).
 //  * k_trsv_generic: any k, one warp per right-hand side through memory.
 //  * k_diag_solve: B(i,c) / A(i,i) for every entry, one thread each.
 #include <climits>
