@@ -104,7 +104,15 @@ int dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, doubl
  * LAPACK does; this is not an error return).
  * Arguments: 1 n >= 0, 2 kl >= 0, 3 ku >= 0, 4 AB, 5 ldab >= 2*kl+ku+1,
  * 6 ipiv (n int32, device), 7 d_info (device).
- * Scratch: none.  NaN entries in a pivot column give unspecified pivots.
+ * Pivot comparisons follow the running-maximum order of LAPACK's IDAMAX: the
+ * running best starts at the first candidate (row j) and a later candidate
+ * replaces it only when its modulus is strictly larger.  So ties go to the
+ * lowest row, and a NaN becomes the pivot only when it is the first candidate
+ * (no later modulus compares larger than a NaN); a NaN below row j is never
+ * chosen over an earlier candidate.
+ * Scratch: for bands wide enough for the multi-CTA kernel, 8 + 8*ceil(n/4)
+ * bytes of hand-off flags from the stream-ordered allocator (cudaMallocAsync
+ * on `stream`, freed in stream order); otherwise none.
  */
 int gbtrf(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *ipiv, int *d_info, cudaStream_t stream);
 
@@ -303,11 +311,14 @@ int dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t strideA
  * 8 (kl, ku), whatever n is; a call needing more returns BANDLU_ERR_SCRATCH.
  * Every GPU that loads the library holds the array until the process exits.
  * The first call on each device resolves the array's device address
- * (cudaGetSymbolAddress) with that device current; make that first call before
- * any stream capture.  All calls share the one array and it keeps the last
- * call's contents (each call clears the pair before detecting), so calls whose
- * work overlaps on the GPU (different streams or threads, no ordering between
- * them) race on it: serialise them.
+ * (cudaGetSymbolAddress) with that device current, and keeps it for that
+ * device's context; after a cudaDeviceReset the next call resolves it again in
+ * the new context.  Make the first call on a device (and the first after a
+ * reset) before any stream capture begins.  Like dispatch_lu, the call
+ * synchronizes `stream` once to read the detected bandwidths.  All calls share
+ * the one array and it keeps the last call's contents (each call clears the pair
+ * before detecting), so calls whose work overlaps on the GPU (different streams
+ * or threads, no ordering between them) race on it: serialise them.
  * Arguments: as dispatch_lu.
  */
 int dispatch_lu_noalloc(const double *A, int64_t n, int64_t lda, double *AB, int64_t ldab, int *ipiv, int *h_kl,

@@ -27,32 +27,45 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "bandlu_oracle.c")
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "liboracle_bandlu.so")
+# Timing build only: the same source compiled with OpenMP, whose pragmas split the
+# detection scan and the conversion over rows/columns and a batch over its
+# matrices.  Nothing in the arithmetic changes (a max-reduction, plain copies and
+# independent matrices); the pinned, checked library is the single-threaded one.
+_OMP_LIB_PATH = os.path.join(_BUILD, "liboracle_bandlu_omp.so")
 _lock = threading.Lock()
 _lib = None
+_omp_lib = None
 
 CFLAGS = ["-O2", "-fPIC", "-shared", "-std=gnu11", "-ffp-contract=off", "-fno-fast-math"]
 
 
-def build(force: bool = False) -> str:
-    """Compile the oracle with gcc into ``oracle/_build``; returns the .so path."""
+def build(force: bool = False, omp: bool = False) -> str:
+    """Compile the oracle with gcc into ``oracle/_build``; returns the .so path.
+    omp=True builds the OpenMP timing variant (used only to time the CPU baseline)."""
     os.makedirs(_BUILD, exist_ok=True)
-    if (not force and os.path.exists(_LIB_PATH)
-            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
-        return _LIB_PATH
-    tmp = _LIB_PATH + f".tmp{os.getpid()}"
-    subprocess.run(["gcc", *CFLAGS, "-o", tmp, _SRC, "-lm"], check=True)
-    os.replace(tmp, _LIB_PATH)
-    return _LIB_PATH
+    path = _OMP_LIB_PATH if omp else _LIB_PATH
+    if (not force and os.path.exists(path)
+            and os.path.getmtime(path) >= os.path.getmtime(_SRC)):
+        return path
+    tmp = path + f".tmp{os.getpid()}"
+    subprocess.run(["gcc", *CFLAGS, *(["-fopenmp"] if omp else []), "-o", tmp, _SRC, "-lm"], check=True)
+    os.replace(tmp, path)
+    return path
 
 
-def _load():
-    global _lib
+def _load(omp: bool = False):
+    global _lib, _omp_lib
     with _lock:
-        if _lib is not None:
+        if omp and _omp_lib is not None:
+            return _omp_lib
+        if not omp and _lib is not None:
             return _lib
-        # A mutation test points this at a deliberately broken build of the oracle to show that
-        # the pins catch the mistake; normal use leaves it unset.
-        path = os.environ.get("BANDLU_ORACLE_LIB") or build()
+        if omp:
+            path = build(omp=True)
+        else:
+            # A mutation test points this at a deliberately broken build of the oracle to show
+            # that the pins catch the mistake; normal use leaves it unset.
+            path = os.environ.get("BANDLU_ORACLE_LIB") or build()
         lib = ctypes.CDLL(path)
         i64, i32, dp, ip = ctypes.c_int64, ctypes.c_int, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)
         i64p = ctypes.POINTER(ctypes.c_int64)
@@ -73,7 +86,10 @@ def _load():
         lib.oracle_diag_solve.argtypes = [i64, dp, i64, i64, dp, i64, ip]
         lib.oracle_classify.argtypes = [i64, i32, i32, i64]
         lib.oracle_dispatch_backslash.argtypes = [dp, i64, i64, dp, i64, i64, dp, i64, ip, ip, ip, ip, ip]
-        _lib = lib
+        if omp:
+            _omp_lib = lib
+        else:
+            _lib = lib
         return lib
 
 
@@ -99,22 +115,22 @@ def ldab_for(kl: int, ku: int) -> int:
     return 2 * kl + ku + 1
 
 
-def detect_bandwidth(A: np.ndarray) -> tuple[int, int]:
-    """(kl, ku) of the n x n row-major matrix held in ``A[:, :n]``."""
+def detect_bandwidth(A: np.ndarray, omp: bool = False) -> tuple[int, int]:
+    """(kl, ku) of the n x n row-major matrix held in ``A[:, :n]`` (omp: the timing build)."""
     A, n, lda = _dense(A)
     kl, ku = ctypes.c_int(), ctypes.c_int()
-    rc = _load().oracle_detect_bandwidth(_dptr(A), n, max(lda, 1), ctypes.byref(kl), ctypes.byref(ku))
+    rc = _load(omp).oracle_detect_bandwidth(_dptr(A), n, max(lda, 1), ctypes.byref(kl), ctypes.byref(ku))
     if rc != 0:
         raise ValueError("oracle_detect_bandwidth: bad argument")
     return kl.value, ku.value
 
 
-def dense_to_band(A: np.ndarray, kl: int, ku: int, ldab: int | None = None) -> np.ndarray:
-    """Band storage of A as an (n, ldab) array: ``AB[j, kl+ku+i-j] = A[i, j]``."""
+def dense_to_band(A: np.ndarray, kl: int, ku: int, ldab: int | None = None, omp: bool = False) -> np.ndarray:
+    """Band storage of A as an (n, ldab) array: ``AB[j, kl+ku+i-j] = A[i, j]`` (omp: the timing build)."""
     A, n, lda = _dense(A)
     ldab = ldab_for(kl, ku) if ldab is None else ldab
     AB = np.empty((n, ldab), dtype=np.float64)
-    rc = _load().oracle_dense_to_band(_dptr(A), n, max(lda, 1), kl, ku, _dptr(AB), ldab)
+    rc = _load(omp).oracle_dense_to_band(_dptr(A), n, max(lda, 1), kl, ku, _dptr(AB), ldab)
     if rc != 0:
         raise ValueError("oracle_dense_to_band: bad argument")
     return AB
@@ -197,8 +213,8 @@ def is_banded(n: int, kl: int, ku: int, ldab: int) -> bool:
     return bool(_load().oracle_is_banded(n, kl, ku, ldab))
 
 
-def dispatch_lu_batched(A: np.ndarray, ldab: int):
-    """Batched dispatch over A of shape (batch, n, lda).
+def dispatch_lu_batched(A: np.ndarray, ldab: int, omp: bool = False):
+    """Batched dispatch over A of shape (batch, n, lda) (omp: the timing build, one matrix per thread).
 
     Returns dict with AB (batch, n, ldab), ipiv (batch, n), kl, ku, info, status
     (0 = factored, 1 = declined by the predicate).
@@ -211,7 +227,7 @@ def dispatch_lu_batched(A: np.ndarray, ldab: int):
     ku = np.zeros(batch, dtype=np.int32)
     info = np.zeros(batch, dtype=np.int32)
     status = np.zeros(batch, dtype=np.int32)
-    _load().oracle_dispatch_lu_batched(_dptr(A), n, max(lda, 1), n * lda, batch, _dptr(AB), ldab, n * ldab,
+    _load(omp).oracle_dispatch_lu_batched(_dptr(A), n, max(lda, 1), n * lda, batch, _dptr(AB), ldab, n * ldab,
                                        _iptr(ipiv), n, _iptr(kl), _iptr(ku), _iptr(info), _iptr(status))
     return dict(AB=AB, ipiv=ipiv, kl=kl, ku=ku, info=info, status=status)
 

@@ -55,6 +55,8 @@ int oracle_detect_bandwidth(const double *A, int64_t n, int64_t lda, int *kl, in
 {
     if (n < 0 || lda < (n > 1 ? n : 1) || !kl || !ku) return -1;
     int64_t best_l = 0, best_u = 0;
+    /* the timing build (-fopenmp) splits the rows over threads; a max-reduction is exact */
+#pragma omp parallel for reduction(max : best_l, best_u) schedule(static)
     for (int64_t i = 0; i < n; ++i) {
         for (int64_t j = 0; j < n; ++j) {
             if (is_nonzero(A[i * lda + j])) {
@@ -80,6 +82,8 @@ int oracle_dense_to_band(const double *A, int64_t n, int64_t lda, int kl, int ku
 {
     if (n < 0 || kl < 0 || ku < 0 || lda < (n > 1 ? n : 1) || ldab < 2 * (int64_t)kl + ku + 1) return -1;
     int64_t kv = (int64_t)kl + ku;
+    /* the timing build (-fopenmp) splits the columns over threads: plain copies */
+#pragma omp parallel for schedule(static)
     for (int64_t j = 0; j < n; ++j) {
         for (int64_t r = 0; r < ldab; ++r) AB[r + j * ldab] = 0.0;
         int64_t i0 = j - ku > 0 ? j - ku : 0;
@@ -380,6 +384,8 @@ void oracle_dispatch_lu_batched(const double *A, int64_t n, int64_t lda, int64_t
                                 double *AB, int64_t ldab, int64_t strideAB, int *ipiv, int64_t strideP,
                                 int *kl, int *ku, int *info, int *status)
 {
+    /* the timing build (-fopenmp) takes one matrix per thread: they are independent */
+#pragma omp parallel for schedule(dynamic, 16)
     for (int64_t b = 0; b < batch; ++b) {
         info[b] = 0;
         status[b] = oracle_dispatch_lu(A + b * strideA, n, lda, AB + b * strideAB, ldab,

@@ -80,6 +80,11 @@ def load():
         lib.bandlu_selftest_div_host.restype = None
         lib.bandlu_selftest_div_device.argtypes = [vp, vp, vp, i64, i32, vp]
         lib.bandlu_selftest_div_device.restype = ctypes.c_int
+        lib.bandlu_peak_dfma.argtypes = [vp, i32, i32, i32, i32, vp]
+        lib.bandlu_peak_dmma.argtypes = [i32, vp, i32, i32, i32, i32, vp]
+        lib.bandlu_peak_hbm_read.argtypes = [vp, i64, vp, i32, vp]
+        for f in ("bandlu_peak_dfma", "bandlu_peak_dmma", "bandlu_peak_hbm_read"):
+            getattr(lib, f).restype = ctypes.c_int
         lib.bandlu_version.restype = ctypes.c_char_p
         lib.bandlu_version.argtypes = []
         _lib = lib
@@ -225,6 +230,21 @@ def bandlu_selftest_div_host(x, d, q, n: int) -> None:
 def bandlu_selftest_div_device(x, d, q, n: int, use_division: int, stream=None) -> int:
     """Self-test hook: the library's known-divisor division (or plain division) on the device."""
     return load().bandlu_selftest_div_device(_ptr(x), _ptr(d), _ptr(q), n, use_division, _stream(stream))
+
+
+def bandlu_peak_dfma(d_sink, blocks: int, threads: int, chains: int, iters: int, stream=None) -> int:
+    """Microbenchmark launch: 2*blocks*threads*chains*iters FP64 flops of independent FMA chains."""
+    return load().bandlu_peak_dfma(_ptr(d_sink), blocks, threads, chains, iters, _stream(stream))
+
+
+def bandlu_peak_dmma(shape: int, d_sink, blocks: int, warps: int, chains: int, iters: int, stream=None) -> int:
+    """Microbenchmark launch: FP64 mma.sync (shape 0 m8n8k4, 1 m16n8k16), chains accumulators per warp."""
+    return load().bandlu_peak_dmma(shape, _ptr(d_sink), blocks, warps, chains, iters, _stream(stream))
+
+
+def bandlu_peak_hbm_read(d_buf, nbytes: int, d_sink, blocks: int, stream=None) -> int:
+    """Microbenchmark launch: one read-only pass over nbytes of device memory."""
+    return load().bandlu_peak_hbm_read(_ptr(d_buf), nbytes, _ptr(d_sink), blocks, _stream(stream))
 
 
 def _ptr_host(x) -> int:

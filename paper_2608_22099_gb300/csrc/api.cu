@@ -22,6 +22,24 @@ bool allow_dynamic_smem(const void *kernel, int bytes) {
   return true;
 }
 
+int device_sms() {
+  constexpr int kMaxDev = 64;
+  static std::mutex mu;
+  static int sms[kMaxDev] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+  if (dev < 0 || dev >= kMaxDev) {
+    int v = 0;
+    return cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0 ? v : 152;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (sms[dev] == 0) {
+    int v = 0;
+    sms[dev] = cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0 ? v : 152;
+  }
+  return sms[dev];
+}
+
 }  // namespace bandlu
 
 namespace {

@@ -229,16 +229,6 @@ __global__ void __launch_bounds__(128) k_batch_factor(long long n, long long bat
   }
 }
 
-int num_sms_b() {
-  static int sms = 0;
-  if (sms == 0) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 152;
-  }
-  return sms;
-}
-
 
 }  // namespace
 
@@ -248,7 +238,7 @@ int launch_batched(const double *A, int64_t n, int64_t lda, int64_t strideA, int
   if (batch == 0) return BANDLU_OK;
   const int vec = ((reinterpret_cast<uintptr_t>(A) & 15u) == 0) && (lda % 2 == 0) && (strideA % 2 == 0);
   long long grid1 = batch;
-  const long long cap = (long long)num_sms_b() * 64;
+  const long long cap = (long long)device_sms() * 64;
   if (grid1 > cap) grid1 = cap;
   k_batch_scan_convert<<<(unsigned)grid1, 256, 0, s>>>(A, n, lda, strideA, batch, AB, ldab, strideAB, d_kl, d_ku,
                                                        d_info, d_status, vec);

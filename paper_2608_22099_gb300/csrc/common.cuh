@@ -117,6 +117,8 @@ namespace bandlu {
 // Opts `kernel` in to `bytes` of dynamic shared memory on the current device,
 // once per (kernel, device) pair; thread-safe.  Returns false if CUDA refuses.
 bool allow_dynamic_smem(const void *kernel, int bytes);
+// Number of SMs of the current device (looked up once per device; thread-safe).
+int device_sms();
 int launch_detect(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t s);
 int launch_dense_to_band(const double *A, int64_t lda, int64_t n, int kl, int ku, double *AB, int64_t ldab,
                          cudaStream_t s);

@@ -33,8 +33,10 @@ __device__ __forceinline__ void block_fold(int lmax, int umax, int *d_kl, int *d
 }
 
 // 16-byte path: A 16-byte aligned and lda even, so every row starts aligned.
-// Vector v of row i holds columns 2v and 2v+1 (2v+1 may be the first padding
-// column when n is odd; it is in bounds because lda >= n+1 then, and ignored).
+// Vector v of row i holds columns 2v and 2v+1.  When n is odd, 2v+1 of the last
+// vector is the first padding column (lda >= n+1 then): it is read, and ignored,
+// on rows 0..n-2, but the last row reads its final column alone with an 8-byte
+// load, so nothing past element (n-1)*lda + n-1 is ever read.
 template <int U>
 __global__ void __launch_bounds__(512) k_detect_vec(const double *__restrict__ A, long long n, long long lda,
                                                     long long nv, long long nseg, int *d_kl, int *d_ku) {
@@ -46,11 +48,18 @@ __global__ void __launch_bounds__(512) k_detect_vec(const double *__restrict__ A
     const long long s = it - i * nseg;
     const ulonglong2 *row = reinterpret_cast<const ulonglong2 *>(A + i * lda);
     const long long v0 = s * seglen + threadIdx.x;
+    // the vector that would reach past the matrix's last element
+    const long long vcut = ((n & 1) && i == n - 1) ? nv - 1 : nv;
     ulonglong2 x[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const long long v = v0 + (long long)u * blockDim.x;
-      x[u] = v < nv ? __ldcs(row + v) : make_ulonglong2(0ull, 0ull);
+      if (v < vcut)
+        x[u] = __ldcs(row + v);
+      else if (v < nv)
+        x[u] = make_ulonglong2(__ldcs(reinterpret_cast<const unsigned long long *>(row + v)), 0ull);
+      else
+        x[u] = make_ulonglong2(0ull, 0ull);
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -92,16 +101,6 @@ __global__ void __launch_bounds__(256) k_detect_scalar(const double *__restrict_
   block_fold(lmax, umax, d_kl, d_ku);
 }
 
-int num_sms() {
-  static int sms = 0;
-  if (sms == 0) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 152;
-  }
-  return sms;
-}
-
 }  // namespace
 
 int launch_detect(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku, cudaStream_t s) {
@@ -112,7 +111,7 @@ int launch_detect(const double *A, int64_t n, int64_t lda, int *d_kl, int *d_ku,
     if (cudaMemsetAsync(d_ku, 0, sizeof(int), s) != cudaSuccess) return BANDLU_ERR_CUDA;
   }
   if (n <= 1) return BANDLU_OK;
-  const int sms = num_sms();
+  const int sms = device_sms();
   const bool vec = ((reinterpret_cast<uintptr_t>(A) & 15u) == 0) && (lda % 2 == 0);
   if (vec) {
     const long long nv = (n + 1) / 2;

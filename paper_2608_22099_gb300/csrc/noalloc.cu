@@ -8,6 +8,8 @@
 // take driver locks or synchronize.  This entry point keeps that scratch in a
 // file-scope __device__ array instead; every GPU that loads the library holds the
 // array (kNoAllocScratchBytes) until the process exits.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -22,27 +24,75 @@ constexpr size_t kNoAllocScratchBytes = sizeof(int) * 64;
 constexpr size_t kNoAllocScratchNeeded = 2 * sizeof(int);  // what one call uses, for every n
 constexpr int kMaxDevices = 64;
 
-std::mutex g_setup_mu;
-int *g_scratch_ptr[kMaxDevices] = {};
+// The array's device address is looked up once per device context: a reset of the
+// device (cudaDeviceReset) ends the context, its module and the array with it, and the
+// next call on that device looks the address up again in the new context.  Contexts are
+// told apart by the driver's unique context id (cuCtxGetId), reached through the
+// runtime's driver entry points so the library needs no link to the driver library.
+typedef CUresult (*PFN_ctxGetCurrent)(CUcontext *);
+typedef CUresult (*PFN_ctxGetId)(CUcontext, unsigned long long *);
 
-// Device address of the scratch array on the current device, resolved once per
-// device with that device current.  Returns nullptr and sets *err on failure.
+struct ScratchCache {
+  int *ptr = nullptr;
+  unsigned long long ctx_id = 0;
+};
+
+std::mutex g_setup_mu;
+ScratchCache g_cache[kMaxDevices];
+bool g_entry_points_tried = false;
+PFN_ctxGetCurrent g_ctx_get_current = nullptr;
+PFN_ctxGetId g_ctx_get_id = nullptr;
+
+// Id of the current device's context, or 0 when the driver cannot report one.
+unsigned long long current_context_id() {
+  if (!g_entry_points_tried) {
+    g_entry_points_tried = true;
+    cudaDriverEntryPointQueryResult q;
+    void *f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_ctx_get_current = reinterpret_cast<PFN_ctxGetCurrent>(f);
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_ctx_get_id = reinterpret_cast<PFN_ctxGetId>(f);
+  }
+  if (g_ctx_get_current == nullptr || g_ctx_get_id == nullptr) return 0;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (g_ctx_get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+  if (g_ctx_get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Device address of the scratch array on the current device, resolved with that
+// device current, once per device context (always, when the context id is not
+// available).  Returns nullptr and sets *err on failure.
 int *scratch_for_current_device(int *err) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
     *err = BANDLU_ERR_CUDA;
     return nullptr;
   }
+  // makes the device's primary context current (initialising it if needed), so the
+  // context id below is the one the launches of this call will run in
+  if (cudaSetDevice(dev) != cudaSuccess) {
+    *err = BANDLU_ERR_CUDA;
+    return nullptr;
+  }
   std::lock_guard<std::mutex> lock(g_setup_mu);
-  if (g_scratch_ptr[dev] == nullptr) {
+  const unsigned long long id = current_context_id();
+  ScratchCache &c = g_cache[dev];
+  if (c.ptr == nullptr || id == 0 || c.ctx_id != id) {
     void *p = nullptr;
     if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
       *err = BANDLU_ERR_CUDA;
       return nullptr;
     }
-    g_scratch_ptr[dev] = static_cast<int *>(p);
+    c.ptr = static_cast<int *>(p);
+    c.ctx_id = id;
   }
-  return g_scratch_ptr[dev];
+  return c.ptr;
 }
 
 }  // namespace

@@ -104,3 +104,18 @@ def make_dense(n: int, kl: int, ku: int, *, dist: str = "uniform", diag_boost: f
 def make_workload(w: Workload, device: str | torch.device = "cpu", lda: int | None = None) -> torch.Tensor:
     return make_dense(w.n, w.kl, w.ku, dist=w.dist, diag_boost=w.diag_boost, seed=w.seed, batch=w.batch,
                       lda=lda, device=device, stray=w.stray)
+
+
+def principal_block(w: Workload, m: int) -> torch.Tensor:
+    """The leading m x m principal block of workload w's matrix, built on the host without
+    the full matrix: the same seeded draw, scattered for rows 0..m-1 with the columns beyond
+    m-1 dropped.  A principal block of a banded matrix is banded with the same (kl, ku)."""
+    if w.batch:
+        raise ValueError("principal_block takes a single-matrix workload")
+    m = min(m, w.n)
+    vals = band_values(w.n, w.kl, w.ku, w.dist, w.seed)[:m]
+    A = torch.zeros((m, m), dtype=torch.float64)
+    scatter_band(A, vals, w.kl, w.ku, w.diag_boost)
+    if w.stray and w.stray[0] < m and w.stray[1] < m:
+        A[w.stray[0], w.stray[1]] = w.stray[2]
+    return A

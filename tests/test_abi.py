@@ -201,6 +201,20 @@ def test_classify_matches_the_oracle(oracle_mod):
         assert bandlu.bandlu_classify(n, kl, ku, ldab) == oracle_mod.classify(n, kl, ku, ldab), (n, kl, ku, ldab)
 
 
+def test_classify_at_the_hand_worked_thresholds():
+    """The library's predicate at the smallest n that takes the band path, worked by hand
+    from the paper's operation counts (tests/golden/predicate_threshold_cases.txt)."""
+    path = os.path.join(ROOT, "tests", "golden", "predicate_threshold_cases.txt")
+    rows = [tuple(int(x) for x in ln.split()) for ln in open(path) if ln.strip() and not ln.startswith("#")]
+    assert len(rows) == 7
+    for kl, ku, n_min in rows:
+        if kl == 0 or ku == 0:
+            continue  # the diagonal and triangular branches come first there
+        ldab = 2 * kl + ku + 1
+        assert bandlu.bandlu_classify(n_min, kl, ku, ldab) == bandlu.KIND_BANDED, (kl, ku, n_min)
+        assert bandlu.bandlu_classify(n_min - 1, kl, ku, ldab) == bandlu.KIND_DENSE, (kl, ku, n_min)
+
+
 @pytest.mark.parametrize("args,expect", [
     ((0, 4, 4, DEV, 4, DEV, DEV, DEV, DEV, DEV), -1),
     ((DEV, -2, 4, DEV, 4, DEV, DEV, DEV, DEV, DEV), -2),

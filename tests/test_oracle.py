@@ -492,6 +492,31 @@ def test_predicate_worked_cases(oracle_mod):
         assert not oracle_mod.is_banded(n, n - 1, n - 1, 10 ** 9)
 
 
+def _threshold_cases():
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "predicate_threshold_cases.txt")
+    rows = []
+    with open(path) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                kl, ku, n_min = (int(x) for x in line.split())
+                rows.append((kl, ku, n_min))
+    return rows
+
+
+def test_predicate_hand_worked_thresholds(oracle_mod):
+    """The smallest n that takes the band path, worked by hand from the operation counts of
+    Eqs. IC-N2, S-N-N3 and D-N3 (tests/golden/predicate_threshold_cases.txt): n_min passes,
+    n_min - 1 and every smaller n decline."""
+    cases = _threshold_cases()
+    assert len(cases) == 7
+    for kl, ku, n_min in cases:
+        ldab = 2 * kl + ku + 1
+        assert oracle_mod.is_banded(n_min, kl, ku, ldab), (kl, ku, n_min)
+        assert not oracle_mod.is_banded(n_min - 1, kl, ku, ldab), (kl, ku, n_min)
+        assert not any(oracle_mod.is_banded(m, kl, ku, ldab) for m in range(max(1, n_min - 50), n_min - 1))
+
+
 def test_predicate_against_exact_rational_cost_model(oracle_mod):
     rng = np.random.default_rng(14)
     for _ in range(2000):

@@ -36,6 +36,8 @@ MUTANTS = [
     ("info_reports_last_zero_pivot", "} else if (info == 0) {\n            info = (int)(j + 1);\n        }\n    }\n#undef AB_",
      "} else {\n            info = (int)(j + 1);\n        }\n    }\n#undef AB_"),
     ("predicate_drops_conversion_cost", "return 3 * (I + C + f) < F3 ? 1 : 0;", "return 3 * (I + f) < F3 ? 1 : 0;"),
+    ("predicate_dense_cost_n_cubed", "__int128 F3 = 2 * N * N * N; /* 3*F */", "__int128 F3 = 3 * N * N * N; /* 3*F */"),
+    ("predicate_fill_width_kl_plus_ku", "__int128 f = N * L * (2 * (L + U) + 1);", "__int128 f = N * L * (L + U + 1);"),
     ("flops_drop_reciprocal", "fl += 1 + km + 2 * km * (ju - j);", "fl += km + 2 * km * (ju - j);"),
     ("dense_lu_swaps_whole_row", "for (int64_t c = j; c < n; ++c) {\n                    double t0 = A[j * lda + c];",
      "for (int64_t c = 0; c < n; ++c) {\n                    double t0 = A[j * lda + c];"),
