@@ -40,8 +40,8 @@ int bandlu_peak_dfma(double *d_sink, int blocks, int threads, int chains, int it
 int bandlu_peak_dmma(int shape, double *d_sink, int blocks, int warps, int chains, int iters, cudaStream_t stream);
 
 /* Read-only HBM stream: reads the `bytes` bytes at d_buf (16-byte aligned,
- * bytes a multiple of 16) once with 16-byte loads that bypass L1 and are
- * evicted first from L2, grid-strided over `blocks` blocks of 512 threads.
+ * bytes a multiple of 16) once with streaming 16-byte loads, in contiguous
+ * 32 KiB chunks dealt round-robin to `blocks` blocks of 512 threads.
  * Work = bytes read.  d_sink: `blocks` 64-bit words (an XOR of what was read). */
 int bandlu_peak_hbm_read(const void *d_buf, int64_t bytes, unsigned long long *d_sink, int blocks,
                          cudaStream_t stream);

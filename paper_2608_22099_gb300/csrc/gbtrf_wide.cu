@@ -37,8 +37,10 @@
 // than any producer can run ahead of its consumer); every wait is bounded.  A wait that gives up raises
 // an error flag that every waiter checks, the kernel ends, and *d_info becomes
 // -BANDLU_ERR_TIMEOUT.
+#include <algorithm>
 #include <climits>
 #include <cstdint>
+#include <cstdlib>
 
 #include "common.cuh"
 #include "rcp.cuh"
@@ -412,15 +414,22 @@ __device__ void factor_panel(const Geo &g, double *blk, int p, double *s_l, Wide
       }
     }
     bar_compute<CW>();
-    // the first largest key over the partials, which are in row order
-    unsigned long long best = sh.key[s][0];
+    // the first largest key over the partials, which are in row order: one lane per
+    // partial and a warp argmax (lowest lane on ties), instead of a serial scan
     int wb = 0;
+    if constexpr (RPT * kCW <= 32) {
+      const unsigned long long kx = lane < RPT * kCW ? sh.key[s][lane] : 0ull;
+      unsigned long long kbest;
+      wb = warp_first_max(kx, &kbest);
+    } else {
+      unsigned long long best = sh.key[s][0];
 #pragma unroll
-    for (int x = 1; x < RPT * kCW; ++x) {
-      const unsigned long long kx = sh.key[s][x];
-      if (kx > best) {
-        best = kx;
-        wb = x;
+      for (int x = 1; x < RPT * kCW; ++x) {
+        const unsigned long long kx = sh.key[s][x];
+        if (kx > best) {
+          best = kx;
+          wb = x;
+        }
       }
     }
     const int p_off = sh.idx[s][wb] - k;
@@ -680,6 +689,392 @@ __global__ void __launch_bounds__(Lay<CW>::kThreads, 1)
   }
 }
 
+// ==== the cluster-pair variant ==================================================
+//
+// GB300's FP64 unit of an SM sub-partition accepts one warp instruction about
+// every 64-76 clocks, whatever the number of active lanes, so the panel CTA's
+// pace is set by the FP64 instructions queued on its four sub-partitions: group
+// A's factor steps and lookahead (26 per row per panel) and group B's lookahead
+// (16 per row per panel), with B's multiply-adds queued in front of A's
+// critical ones.  Here group B runs on its own SM, CTA 1 of a two-CTA cluster:
+//
+//  * CTA 0 (A): group A factors panel p and applies it to block p+1, as above,
+//    keeping the last kRB panels' multipliers and pivots in a ring in shared
+//    memory.  A storer warp writes finished panels to AB, publishes them, and
+//    tells CTA 1 that panel p's multipliers are ready; CTA 1 reads them from the
+//    ring through distributed shared memory and returns the entry when done.
+//  * CTA 1 (B): group B applies panel q to block q+2 and sends that block into
+//    CTA 0's shared memory (where it arrives as block p+1 of panel p = q+1)
+//    (and, with kHand = 4, then applies panel q to block q+3).  A loader warp
+//    brings each block in from AB (a bulk copy once its update CTA hands it
+//    over, else a fresh load).
+//  * CTAs 2.. (update CTAs) own the blocks b >= kHand round-robin, apply panels
+//    p_first(b)..b-kHand and hand the block over (block_ready[b]).
+//
+// Every element still receives the unblocked elimination's fma sequence in the
+// same order (panels are applied to a block in increasing order by whichever CTA
+// holds it), so the factors are bit-identical.  Cross-CTA data moves with plain
+// loads and stores through distributed shared memory; after its stores each warp
+// (or the one signalling thread, after the group's barrier) arrives with release
+// semantics at cluster scope on the receiving CTA's mbarrier, and the receivers
+// wait on it with acquire at cluster scope.  Group A's own path has no remote
+// operation.  Nothing is asynchronous between the two CTAs, so when both have
+// passed the final cluster barrier no transfer is in flight.
+// Every wait is bounded, as in the single-CTA panel kernel.
+
+constexpr int kRB = 4;      // multiplier ring entries (panels) on CTA 0
+constexpr int kBBufs = 4;   // block buffers on CTA 1
+// Update CTAs apply panels p_first(b)..b-kHand to block b and hand it over; CTA 1
+// applies panels b-kHand+1..b-2 (one per panel period for each value of kHand - 2).
+constexpr int kHand = 3;
+
+template <int CW>
+struct PairShared {
+  WideShared<CW, 1> w;
+  unsigned long long mb_mult[kRB];     // CTA 1: panel q factored, its multipliers in CTA 0's ring (1 arrival, storer)
+  unsigned long long mb_credit[kRB];   // CTA 0: CTA 1 has read ring entry q % kRB (1 arrival)
+  unsigned long long mb_blk[kRing];    // CTA 0: block b arrived in buf(b), event b-2 (one arrival per warp of B)
+  unsigned long long mb_afree[kRing];  // CTA 1: CTA 0's buffer of panel p stored, event p (1 arrival, storer)
+  unsigned long long mb_bload[kBBufs]; // CTA 1: block b in its buffer, event b-2 (loader)
+  unsigned long long mb_bsent[kBBufs]; // CTA 1: block b sent, its buffer free, event b-2 (group B)
+  int rpk[kRB][kNB];                   // CTA 0: pivot offsets of the ring's panels (read by CTA 1)
+  int rzp[kRB][kNB];                   // CTA 0: exact-zero-pivot flags of the ring's panels
+};
+
+__device__ __forceinline__ unsigned cl_map(const void *p, unsigned rank) {
+  unsigned r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(rank));
+  return r;
+}
+// Generic address of the same shared-memory object in CTA `rank` of the cluster;
+// ordinary loads and stores through it reach that CTA's shared memory.
+template <class T>
+__device__ __forceinline__ T *cl_generic(T *p, unsigned rank) {
+  unsigned long long r;
+  asm volatile("mapa.u64 %0, %1, %2;" : "=l"(r) : "l"(reinterpret_cast<unsigned long long>(p)), "r"(rank));
+  return reinterpret_cast<T *>(r);
+}
+__device__ __forceinline__ void cl_st2(unsigned raddr, double a, double b) {
+  asm volatile("st.shared::cluster.v2.f64 [%0], {%1, %2};" ::"r"(raddr), "d"(a), "d"(b) : "memory");
+}
+__device__ __forceinline__ void cl_st1(unsigned raddr, double a) {
+  asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(raddr), "d"(a) : "memory");
+}
+// One arrival on an mbarrier of CTA `rank`, ordering this thread's earlier
+// memory operations before it at cluster scope.
+__device__ __forceinline__ void cl_arrive(const unsigned long long *bar, unsigned rank) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cl_map(bar, rank)) : "memory");
+}
+__device__ __forceinline__ bool cl_try_wait(unsigned long long *bar, unsigned parity) {
+  unsigned ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ void cluster_barrier() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ unsigned ring_parity(int e, int R) { return (unsigned)(e / R) & 1u; }
+
+// Blocks b >= kHand pass through an update CTA, which applies panels p_first(b)..b-kHand.
+__device__ __forceinline__ bool handed_off_pair(const Geo &g, int b) {
+  return b >= kHand && p_first(g, b) <= b - kHand;
+}
+
+template <int CW>
+__global__ void __launch_bounds__(32 * (CW + 1), 1)
+    k_gbtrf_wide_pair(Geo g, double *__restrict__ AB, int *__restrict__ ipiv, int *__restrict__ d_info,
+                      int *__restrict__ flags) {
+  constexpr int kCT = Lay<CW>::kCT, kCW = CW;
+  extern __shared__ __align__(16) double smem[];
+  __shared__ PairShared<CW> ps;
+  WideShared<CW, 1> &sh = ps.w;
+  int *err = flags;
+  int *panel_ready = flags + 2;
+  int *block_ready = flags + 2 + g.npan;
+  const long long bsz = (long long)kNB * g.ldab;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // CTA 0: kPanelBufs block buffers and a ring of kRB panels of multipliers; CTA 1: kBBufs
+  // block buffers; update CTAs: kMaxActive block buffers
+  double *blocks = smem;
+  double *s_lbase = smem + (size_t)kPanelBufs * bsz;
+  auto buf = [&](int b) { return blocks + (long long)(b % kPanelBufs) * bsz; };
+  auto bbuf = [&](int b) { return blocks + (long long)((b - 2) % kBBufs) * bsz; };
+  auto mults = [&](int q) { return s_lbase + (size_t)(q % kRB) * kNB * g.kl; };
+
+  if (tid == 0) {
+    for (int i = 0; i < kRing; ++i) {
+      mbar_init(&sh.mb_done[i], 1);
+      mbar_init(&sh.mb_stored[i], 1);
+      mbar_init(&ps.mb_blk[i], kCW);
+      mbar_init(&ps.mb_afree[i], 1);
+    }
+    for (int i = 0; i < kRB; ++i) {
+      mbar_init(&ps.mb_mult[i], 1);
+      mbar_init(&ps.mb_credit[i], 1);
+    }
+    for (int i = 0; i < kBBufs; ++i) {
+      mbar_init(&ps.mb_bload[i], 1);
+      mbar_init(&ps.mb_bsent[i], 1);
+    }
+    sh.info = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  cluster_barrier();  // every CTA's barriers initialised before any remote arrival
+
+  // bounded waits (all threads of a compute group, or one warp)
+  auto grp_wait_cl = [&](unsigned long long *bar, unsigned par, int bar_id) -> bool {
+    if (tid == 0) sh.ok[0] = bounded_poll([&] { return cl_try_wait(bar, par); }, err) ? 1 : 0;
+    bar_group<CW>(bar_id);
+    const bool ok = sh.ok[0] != 0;
+    bar_group<CW>(bar_id);
+    return ok;
+  };
+  auto grp_wait_local = [&](unsigned long long *bar, unsigned par, int bar_id) -> bool {
+    if (tid == 0) sh.ok[0] = bounded_poll([&] { return mbar_try_wait(bar, par); }, err) ? 1 : 0;
+    bar_group<CW>(bar_id);
+    const bool ok = sh.ok[0] != 0;
+    bar_group<CW>(bar_id);
+    return ok;
+  };
+
+  if (blockIdx.x == 0) {
+    if (warp < kCW) {
+      // ---------------- CTA 0, group A: factorisation of panel p, lookahead to block p+1 ----------------
+      int info = 0, bpar = 0;
+      load_block(g, AB, buf(0), 0, true, tid, kCT);
+      if (g.npan > 1) load_block(g, AB, buf(1), 1, true, tid, kCT);
+      bar_compute<CW>();
+      for (int p = 0; p < g.npan; ++p) {
+        // ring entry p % kRB last held panel p - kRB, which CTA 1 reads: wait until it has
+        if (p >= kRB && p - kRB + 2 < g.npan &&
+            !grp_wait_cl(&ps.mb_credit[p % kRB], ring_parity(p - kRB, kRB), kBarA))
+          break;
+        factor_panel<CW, 1>(g, buf(p), p, mults(p), sh, bpar, info);
+        if (tid == 0) {
+          sh.info = info;
+#pragma unroll
+          for (int k = 0; k < kNB; ++k) {
+            sh.pvr[p % kRing][k] = sh.pk[p & 1][k];
+            ps.rpk[p % kRB][k] = sh.pk[p & 1][k];
+            ps.rzp[p % kRB][k] = sh.zp[p & 1][k];
+          }
+        }
+        bar_compute<CW>();
+        if (tid == 0) mbar_arrive(&sh.mb_done[p % kRing]);  // the storer (which also tells CTA 1)
+        double lr[1][kNB];
+        panel_multipliers<CW, 1>(g, mults(p), p, tid, lr);
+        if (p + 1 < g.npan) {
+          const int b = p + 1;
+          if (b >= 2 && !grp_wait_cl(&ps.mb_blk[(b - 2) % kRing], ring_parity(b - 2, kRing), kBarA)) break;
+          if (p >= p_first(g, b)) {  // uniform
+            apply_panel<CW, 1>(g, buf(b), b, p, lr, sh.pk[p & 1], sh.zp[p & 1], sh.bc[0], tid, kBarA, bpar);
+            bar_compute<CW>();
+          }
+        }
+      }
+    } else if (warp == kCW) {
+      // ---------------- CTA 0, storer: finished panels to AB, published ----------------
+      for (int p = 0; p < g.npan; ++p) {
+        unsigned long long *mb = &sh.mb_done[p % kRing];
+        if (!io_wait([&] { return mbar_try_wait(mb, ring_parity(p, kRing)); }, err)) break;
+        // CTA 1 applies panel p to blocks p+2 and p+3: its multipliers and pivots are
+        // in the ring (ordered before group A's arrival on mb_done, which this warp acquired)
+        if (p + 2 < g.npan && lane == 0) cl_arrive(&ps.mb_mult[p % kRB], 1);
+        const int c0 = p * kNB, nc = min(kNB, g.n - c0);
+        const double *src = buf(p);
+        double *dst = AB + (long long)c0 * g.ldab;
+        const int ld = (int)g.ldab;
+        for (int k = 0; k < nc; ++k)
+          for (int rr = g.kv + lane; rr <= g.kv + g.kl; rr += 32) dst[k * ld + rr] = src[k * ld + rr];
+        if (lane < nc) ipiv[c0 + lane] = c0 + lane + sh.pvr[p % kRing][lane] + 1;
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) st_release(panel_ready + p, 1);
+        store_block(g, AB, src, p, lane, 32);
+        __syncwarp();
+        // this buffer takes block p+3 next, which CTA 1 sends
+        if (p + 3 < g.npan && lane == 0) cl_arrive(&ps.mb_afree[p % kRing], 1);
+      }
+      if (lane == 0) *d_info = ld_acquire(err) ? -BANDLU_ERR_TIMEOUT : sh.info;
+    }
+  } else if (blockIdx.x == 1) {
+    if (warp < kCW) {
+      // ---------------- CTA 1, group B: panel q to blocks q+2 (sent to CTA 0) and q+3 ----------------
+      int bpar = 0;
+      bool ok = true;
+      for (int q = 0; ok && q + 2 < g.npan; ++q) {
+        if (!grp_wait_cl(&ps.mb_mult[q % kRB], ring_parity(q, kRB), kBarB)) break;
+        // panel q's multipliers and pivots, read from CTA 0's ring
+        double lr[1][kNB];
+        panel_multipliers<CW, 1>(g, cl_generic(mults(q), 0), q, tid, lr);
+        int pk[kNB], zp[kNB];
+        const int *rpk = cl_generic(&ps.rpk[q % kRB][0], 0), *rzp = cl_generic(&ps.rzp[q % kRB][0], 0);
+#pragma unroll
+        for (int k = 0; k < kNB; ++k) {
+          pk[k] = rpk[k];
+          zp[k] = rzp[k];
+        }
+        bar_group<CW>(kBarB);
+        if (tid == 0) cl_arrive(&ps.mb_credit[q % kRB], 0);  // ring entry read: CTA 0 may refill it
+        for (int which = 0; which <= kHand - 3; ++which) {
+          const int b = q + 2 + which;
+          if (b >= g.npan) break;
+          // block b's first use here (panel b-kHand+1, or panel 0): wait for the loader
+          if (q == max(0, b - kHand + 1)) {
+            if (!grp_wait_local(&ps.mb_bload[(b - 2) % kBBufs], ring_parity(b - 2, kBBufs), kBarB)) {
+              ok = false;
+              break;
+            }
+          }
+          if (q >= p_first(g, b)) {  // uniform
+            apply_panel<CW, 1>(g, bbuf(b), b, q, lr, pk, zp, sh.bc[1], tid, kBarB, bpar);
+            bar_group<CW>(kBarB);
+          }
+          if (which == 0) {
+            // CTA 0's buffer of block b held panel b-3: wait until its storer is done with it
+            if (b >= 3 && !grp_wait_cl(&ps.mb_afree[(b - 3) % kRing], ring_parity(b - 3, kRing), kBarB)) {
+              ok = false;
+              break;
+            }
+            const double *s = bbuf(b);
+            const double *d = buf(b);
+            const int tot = kNB * (int)g.ldab;
+            for (int e = 2 * tid; e + 1 < tot; e += 2 * kCT) cl_st2(cl_map(d + e, 0), s[e], s[e + 1]);
+            if ((tot & 1) && tid == 0) cl_st1(cl_map(d + tot - 1, 0), s[tot - 1]);
+            __syncwarp();
+            if (lane == 0) cl_arrive(&ps.mb_blk[(b - 2) % kRing], 0);  // one arrival per warp
+            bar_group<CW>(kBarB);
+            if (tid == 0) mbar_arrive(&ps.mb_bsent[(b - 2) % kBBufs]);  // the buffer may take block b+4
+          }
+        }
+      }
+    } else if (warp == kCW) {
+      // ---------------- CTA 1, loader: blocks b >= 2 into its buffers ----------------
+      for (int b = 2; b < g.npan; ++b) {
+        const int e = b - 2;
+        if (e >= kBBufs) {  // the buffer held block b-4, sent to CTA 0 by now
+          unsigned long long *mb = &ps.mb_bsent[e % kBBufs];
+          const unsigned par = ring_parity(e - kBBufs, kBBufs);
+          if (!io_wait([&] { return mbar_try_wait(mb, par); }, err)) break;
+        }
+        double *dst = bbuf(b);
+        unsigned long long *ml = &ps.mb_bload[e % kBBufs];
+        if (handed_off_pair(g, b)) {
+          const int *f = block_ready + b;
+          if (!io_wait([&] { return ld_acquire(f) != 0; }, err)) break;
+          if (g.vec && (b + 1) * kNB <= g.n) {
+            if (lane == 0) bulk_prefetch_block(g, AB, dst, b, ml);  // completes the phase itself
+            __syncwarp();
+            continue;
+          }
+          if (g.vec) {
+            io_prefetch_block(g, AB, dst, b);
+          } else {
+            load_block(g, AB, dst, b, false, lane, 32);
+          }
+        } else {
+          load_block(g, AB, dst, b, true, lane, 32);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(ml);
+      }
+    }
+  } else {
+    // ---------------- update CTAs: panels p_first(b)..b-kHand to their blocks ----------------
+    if (warp >= kCW) return;
+    const int G = gridDim.x - 2, u = blockIdx.x - 2;
+    int bpar = 0;
+    for (int p = 0; p + kHand < g.npan; ++p) {
+      const int lo = p + kHand, hi = b_last(g, p);
+      const int b0 = lo + ((u - (lo - kHand)) % G + G) % G;
+      if (b0 > hi) continue;
+      const int *f = panel_ready + p;
+      if (!compute_wait<CW, 1>([&] { return ld_acquire(f) != 0; }, err, sh)) break;
+      const int c0q = p * kNB, ncq = min(kNB, g.n - c0q);
+      if (tid < kNB) {
+        const int k = tid;
+        sh.pk[0][k] = k < ncq ? __ldcg(ipiv + c0q + k) - 1 - (c0q + k) : 0;
+        sh.zp[0][k] = k < ncq ? (nz(__ldcg(AB + (long long)(c0q + k) * g.ldab + g.kv)) ? 0 : 1) : 1;
+      }
+      double lr[1][kNB];
+#pragma unroll
+      for (int k = 0; k < kNB; ++k) {
+        const int t = tid - k;
+        lr[0][k] = (k < ncq && t >= 1 && t <= min(g.kl, g.n - 1 - (c0q + k)))
+                       ? __ldcg(AB + (long long)(c0q + k) * g.ldab + g.kv + t)
+                       : 0.0;
+      }
+      bar_compute<CW>();
+      for (int b = b0; b <= hi; b += G) {
+        double *blk = blocks + (long long)(((b - kHand) / G) % kMaxActive) * bsz;
+        if (p == p_first(g, b)) {
+          load_block(g, AB, blk, b, true, tid, kCT);
+          bar_compute<CW>();
+        }
+        apply_panel<CW, 1>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh.bc[0], tid, kBarA, bpar);
+        bar_compute<CW>();
+        if (p == b - kHand) {
+          store_block(g, AB, blk, b, tid, kCT);
+          __threadfence();
+          bar_compute<CW>();
+          if (tid == 0) st_release(block_ready + b, 1);
+        }
+      }
+    }
+    return;
+  }
+  // the cluster's two CTAs leave together: no distributed-shared-memory access can
+  // reach a CTA that has exited
+  cluster_barrier();
+}
+
+template <int CW>
+int launch_pair(const Geo &g, int grid, size_t smem, double *AB, int *ipiv, int *d_info, int *flags, cudaStream_t s) {
+  constexpr int kThreads = 32 * (CW + 1);
+  if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_wide_pair<CW>), 200 * 1024)) return BANDLU_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 2;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  at[1].id = cudaLaunchAttributeCooperative;
+  at[1].val.cooperative = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, k_gbtrf_wide_pair<CW>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return BANDLU_NOT_BANDED;
+  }
+  if (clusters * 2 < grid) return BANDLU_NOT_BANDED;
+  cfg.numAttrs = 2;
+  Geo gg = g;
+  if (cudaLaunchKernelEx(&cfg, k_gbtrf_wide_pair<CW>, gg, AB, ipiv, d_info, flags) != cudaSuccess)
+    return BANDLU_ERR_CUDA;
+  return BANDLU_OK;
+}
+
+// BANDLU_WIDE_SINGLE=1 in the environment selects the single-CTA panel kernel
+// for every shape (read once): the comparison the cluster pair is measured against.
+bool pair_disabled() {
+  static const bool off = [] {
+    const char *v = std::getenv("BANDLU_WIDE_SINGLE");
+    return v != nullptr && v[0] == '1';
+  }();
+  return off;
+}
+
 // Returns BANDLU_OK after a launch, BANDLU_NOT_BANDED when the kernel cannot be
 // made resident (the caller then takes another kernel), or BANDLU_ERR_CUDA.
 template <int CW, int RPT>
@@ -741,8 +1136,26 @@ int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *
     cudaFreeAsync(flags, s);
     return BANDLU_ERR_CUDA;
   }
-  int rc;
-  if (cw == 2)
+  int rc = BANDLU_NOT_BANDED;
+  if (rpt == 1 && sms >= 4 && !pair_disabled()) {
+    // the cluster pair: CTA 0 factors, CTA 1 runs the second lookahead group
+    const int grid2 = sms & ~1;
+    const size_t need_a = (size_t)kPanelBufs * kNB * (size_t)ldab + (size_t)kRB * kNB * kl;
+    const size_t need_b = (size_t)kBBufs * kNB * (size_t)ldab;
+    const size_t need_u = (size_t)kMaxActive * kNB * (size_t)ldab;
+    const size_t smem2 = std::max(need_a, std::max(need_b, need_u)) * sizeof(double);
+    if (smem2 <= 200 * 1024 && span <= (long long)kMaxActive * (grid2 - 2)) {
+      if (cw == 2)
+        rc = launch_pair<2>(g, grid2, smem2, AB, ipiv, d_info, flags, s);
+      else if (cw == 4)
+        rc = launch_pair<4>(g, grid2, smem2, AB, ipiv, d_info, flags, s);
+      else
+        rc = launch_pair<9>(g, grid2, smem2, AB, ipiv, d_info, flags, s);
+    }
+  }
+  if (rc != BANDLU_NOT_BANDED) {
+    // launched (or failed): nothing more to do
+  } else if (cw == 2)
     rc = launch_rpt<2, 1>(g, sms, smem, AB, ipiv, d_info, flags, s);
   else if (cw == 4)
     rc = launch_rpt<4, 1>(g, sms, smem, AB, ipiv, d_info, flags, s);

@@ -83,24 +83,30 @@ __global__ void k_peak_dmma_m16n8k16(double *__restrict__ sink, int iters) {
   else if (s == -1.0) sink[blockIdx.x] = s;
 }
 
+// Each block reads contiguous chunks of 512 x 4 16-byte vectors (32 KiB), chunk c
+// by block c mod gridDim: every warp load is one contiguous 512-byte run.
 __global__ void __launch_bounds__(512) k_peak_read(const ulonglong2 *__restrict__ p, long long nvec,
                                                    unsigned long long *__restrict__ sink) {
+  constexpr int U = 4;
   __shared__ unsigned long long acc;
   if (threadIdx.x == 0) acc = 0ull;
   __syncthreads();
   unsigned long long x = 0ull;
-  const long long stride = (long long)gridDim.x * blockDim.x;
-  long long v = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  for (; v + 3 * stride < nvec; v += 4 * stride) {
-    const ulonglong2 a = __ldcs(p + v), b = __ldcs(p + v + stride), c = __ldcs(p + v + 2 * stride),
-                     d = __ldcs(p + v + 3 * stride);
-    x ^= a.x ^ a.y ^ b.x ^ b.y ^ c.x ^ c.y ^ d.x ^ d.y;
+  const long long chunk = (long long)blockDim.x * U;
+  const long long nchunks = (nvec + chunk - 1) / chunk;
+  for (long long c = blockIdx.x; c < nchunks; c += gridDim.x) {
+    const long long v0 = c * chunk + threadIdx.x;
+    ulonglong2 a[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const long long v = v0 + (long long)u * blockDim.x;
+      a[u] = v < nvec ? __ldcs(p + v) : make_ulonglong2(0ull, 0ull);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) x ^= a[u].x ^ a[u].y;
   }
-  for (; v < nvec; v += stride) {
-    const ulonglong2 a = __ldcs(p + v);
-    x ^= a.x ^ a.y;
-  }
-  const unsigned lo = __reduce_xor_sync(bandlu::FULL, (unsigned)x), hi = __reduce_xor_sync(bandlu::FULL, (unsigned)(x >> 32));
+  const unsigned lo = __reduce_xor_sync(bandlu::FULL, (unsigned)x),
+                 hi = __reduce_xor_sync(bandlu::FULL, (unsigned)(x >> 32));
   if ((threadIdx.x & 31) == 0) atomicXor(&acc, ((unsigned long long)hi << 32) | lo);
   __syncthreads();
   if (threadIdx.x == 0) sink[blockIdx.x] = acc;
