@@ -418,8 +418,21 @@ def measure_single(torch, bandlu, w, dev, stream, flush, reps: int, fp64_peak: f
     t_disp = statistics.median(event_ms(torch, stream, disp, reps, flush)) * 1e-3
     t_det = statistics.median(event_ms(torch, stream, det, reps, flush)) * 1e-3
     rc, dkl, dku = res["rc"]
+    # the same dispatch with the decision on the device (no host round trip)
+    sc = torch.zeros(4, dtype=torch.int32, device=dev)
+    ABa = torch.zeros_like(AB)
+    ipa = torch.zeros_like(ipiv)
+
+    def dasync():
+        bandlu.check(bandlu.dispatch_lu_async(A, n, n, ABa, ldab, ipa, sc[0:1], sc[1:2], sc[2:3], sc[3:4], stream),
+                     "dispatch_lu_async")
+    t_async = statistics.median(event_ms(torch, stream, dasync, reps, flush)) * 1e-3
+    if tuple(int(v) for v in sc[:3].cpu()) != (dkl, dku, rc) or (rc == 0 and not torch.equal(ABa, AB)):
+        raise RuntimeError(f"{w.name}: dispatch_lu_async disagrees with dispatch_lu")
+    del ABa, ipa
     det_bytes = 8.0 * n * n
     out = {"status": rc, "detected_kl": dkl, "detected_ku": dku, "dispatch_ms": t_disp * 1e3,
+           "dispatch_async_ms": t_async * 1e3,
            "detect_us": t_det * 1e6, "detect_gbs": det_bytes / t_det / 1e9,
            "detect_frac_hbm": det_bytes / t_det / 1e9 / hbm_peak}
     if rc == 0:
@@ -604,6 +617,20 @@ def run_ours(args):
     ms_per_step = multirank.max_over_ranks(sum(step_ms), device=dev) / args.steps
     value = multirank.job_throughput(multirank.sum_over_ranks(flops, device=dev), ms_per_step * 1e-3) / 1e9
 
+    # the same step with the decision on the device (dispatch_lu_async: no host round trip;
+    # its factorisation is the same multi-CTA kernel, enqueued before the bandwidths are known)
+    sc = torch.zeros(4, dtype=torch.int32, device=dev)
+    AB3 = torch.zeros_like(AB)
+    ipiv3 = torch.zeros_like(ipiv)
+
+    def step_async():
+        bandlu.check(bandlu.dispatch_lu_async(A, n, n, AB3, ldab, ipiv3, sc[0:1], sc[1:2], sc[2:3], sc[3:4], stream),
+                     "dispatch_lu_async")
+    async_ms = statistics.mean(event_ms(torch, stream, step_async, max(3, min(args.steps, 10)), flush))
+    if tuple(int(v) for v in sc.cpu()) != (kl, ku, 0, 0) or not torch.equal(AB3, AB):
+        raise RuntimeError("dispatch_lu_async disagrees with dispatch_lu")
+    del AB3, ipiv3
+
     # stage breakdown through the same C ABI, CUDA events on the launching stream
     reps = max(3, min(args.steps, 10))
     klku = torch.zeros(2, dtype=torch.int32, device=dev)
@@ -729,7 +756,7 @@ def run_ours(args):
                              "l2": "inputs (8 GiB) larger than L2, and L2 flushed between steps (512 MiB write, "
                                    "then a 256 MiB read)",
                              "parallelism": "replicas" if world > 1 else "single"},
-            "dispatch_ms": ms_per_step, "flops_per_step": flops, "stages": stages,
+            "dispatch_ms": ms_per_step, "dispatch_async_ms": async_ms, "flops_per_step": flops, "stages": stages,
             "dense_lu_ms_estimate": dense_est,
             "dense_lu_estimate_from": "cuSOLVER getrf (torch) timed at n=16384 on this GPU, x (32768/16384)^3",
             "speedup_over_dense_estimate": (dense_est / ms_per_step) if dense_est else None,
@@ -823,9 +850,8 @@ def run_workload_report(args):
         t_disp = timed(disp, reps)
         t_det = timed(det, reps)
         # the same dispatch with the decision on the device (no host round trip), and that call
-        # captured once in a CUDA graph and replayed; for the bands its one-CTA kernels cover
-        # (wider bands take its block-wide fallback, seconds at n = 32768)
-        if kl <= 27 and 2 * kl + ku + 1 <= 256:
+        # captured once in a CUDA graph and replayed
+        if True:
             sc = torch.zeros(4, dtype=torch.int32, device=dev)
 
             def dasync(st):

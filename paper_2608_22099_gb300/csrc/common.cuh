@@ -105,6 +105,15 @@ __host__ __device__ inline bool predicate_banded(long long n, long long kl, long
   return lhs < 2 * N * N * N;
 }
 
+// The cluster-pair wide factorisation takes a band (whose window factorisation
+// path is the generic one) when its panels of kl + 4 rows fit the compute group of
+// `rows_cap` threads the kernel was launched with (0: not launched) and the band
+// spans at least two 4-column blocks (n >= 16, kl >= 1, kl + ku >= 8).  The
+// device-side dispatch and the kernel both apply this rule.
+__host__ __device__ inline bool wide_pair_takes(long long n, int kl, int ku, int rows_cap) {
+  return rows_cap > 0 && n >= 16 && kl >= 1 && (long long)kl + ku >= 8 && kl + 4 <= rows_cap;
+}
+
 }  // namespace bandlu
 
 #define BANDLU_CHECK_LAUNCH()                         \
@@ -139,6 +148,23 @@ int launch_decide_convert(const double *A, int64_t lda, int64_t n, int64_t ldab,
                           int *d_status, double *AB, cudaStream_t s);
 int launch_gbtrf_on_device(int64_t n, double *AB, int64_t ldab, int *ipiv, const int *d_kl, const int *d_ku,
                            const int *d_status, int *d_info, cudaStream_t s);
+// dispatch_lu_async's wide path: the cluster-pair kernel enqueued with the band
+// storage's largest admissible kl ((ldab-1)/2) before (kl, ku) are known.
+// prepare: when that kernel can be made resident for this ldab, takes and clears
+// its hand-off flags (stream-ordered) and sets *rows_cap > 0 and *flags; else
+// *rows_cap = 0.  launch: enqueues the kernel (which reads (kl, ku) and the
+// decision flags[1] on the device and exits unless the band is its) and frees the
+// flags.
+struct WideDeferred {
+  int rows_cap = 0;
+  int cw = 0;
+  int grid = 0;
+  size_t smem = 0;
+  int *flags = nullptr;
+};
+int prepare_gbtrf_wide_deferred(int64_t n, int64_t ldab, cudaStream_t s, WideDeferred *wd);
+int launch_gbtrf_wide_deferred(const WideDeferred &wd, int64_t n, double *AB, int64_t ldab, int *ipiv,
+                               const int *d_kl, const int *d_ku, int *d_info, cudaStream_t s);
 // d_info: when not null and *d_info != 0 (a singular factor), B is left as it is.
 int launch_gbtrs(int64_t n, int kl, int ku, int64_t nrhs, const double *AB, int64_t ldab, const int *ipiv, double *B,
                  int64_t ldb, const int *d_info, cudaStream_t s);

@@ -545,7 +545,8 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_on_device(int n, doubl
                                                                      const int *__restrict__ d_kl,
                                                                      const int *__restrict__ d_ku,
                                                                      const int *__restrict__ d_status,
-                                                                     int *__restrict__ d_info, size_t smem_bytes) {
+                                                                     int *__restrict__ d_info, size_t smem_bytes,
+                                                                     int wide_rows_cap, int *__restrict__ wide_flag) {
   extern __shared__ double W[];
   __shared__ WinShared sh;
   if (*d_status != BANDLU_OK) return;  // declined: nothing is written
@@ -554,6 +555,11 @@ __global__ void __launch_bounds__(kWarps * 32, 1) k_gbtrf_on_device(int n, doubl
   size_t smem = 0;
   int path = factor_path(n, kl, ku, ldab, &K, &PF, &smem);
   if (path == 1 && smem > smem_bytes) path = 2;
+  if (path == 2 && wide_flag != nullptr && wide_pair_takes(n, kl, ku, wide_rows_cap)) {
+    // the cluster-pair kernel enqueued after this one factors the band
+    if (threadIdx.x == 0) *wide_flag = 1;
+    return;
+  }
   if (path == 0) {
     if (threadIdx.x < 32) regwin_factor(n, kl, ku, AB, (int)ldab, ipiv, d_info);
   } else if (path == 1) {
@@ -628,8 +634,20 @@ int launch_gbtrf_on_device(int64_t n, double *AB, int64_t ldab, int *ipiv, const
   const long long cs = ldab < 256 ? ldab : 256;
   const size_t smem = (size_t)((kWinMaxKl + 1 + kDelta) * cs) * sizeof(double);
   if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_on_device), 200 * 1024)) return BANDLU_ERR_CUDA;
-  k_gbtrf_on_device<<<1, kWarps * 32, smem, s>>>((int)n, AB, ldab, ipiv, d_kl, d_ku, d_status, d_info, smem);
-  BANDLU_CHECK_LAUNCH();
+  // a band storage that admits kl >= kWinMaxKl + 1 may hold a band no window takes:
+  // the multi-CTA kernel is enqueued too and runs only if the decision on the device is its
+  WideDeferred wd;
+  if (ldab >= 2 * (kWinMaxKl + 1) + 1) {
+    const int rc = prepare_gbtrf_wide_deferred(n, ldab, s, &wd);
+    if (rc != BANDLU_OK) return rc;
+  }
+  k_gbtrf_on_device<<<1, kWarps * 32, smem, s>>>((int)n, AB, ldab, ipiv, d_kl, d_ku, d_status, d_info, smem,
+                                                 wd.rows_cap, wd.flags != nullptr ? wd.flags + 1 : nullptr);
+  if (cudaPeekAtLastError() != cudaSuccess) {
+    if (wd.flags != nullptr) cudaFreeAsync(wd.flags, s);
+    return BANDLU_ERR_CUDA;
+  }
+  if (wd.rows_cap > 0) return launch_gbtrf_wide_deferred(wd, n, AB, ldab, ipiv, d_kl, d_ku, d_info, s);
   return BANDLU_OK;
 }
 

@@ -41,6 +41,9 @@
 #include <climits>
 #include <cstdint>
 #include <cstdlib>
+#include <map>
+#include <mutex>
+#include <tuple>
 
 #include "common.cuh"
 #include "rcp.cuh"
@@ -788,9 +791,19 @@ __device__ __forceinline__ bool handed_off_pair(const Geo &g, int b) {
 
 template <int CW>
 __global__ void __launch_bounds__(32 * (CW + 1), 1)
-    k_gbtrf_wide_pair(Geo g, double *__restrict__ AB, int *__restrict__ ipiv, int *__restrict__ d_info,
-                      int *__restrict__ flags) {
+    k_gbtrf_wide_pair(Geo g0, double *__restrict__ AB, int *__restrict__ ipiv, int *__restrict__ d_info,
+                      int *__restrict__ flags, const int *__restrict__ d_kl, const int *__restrict__ d_ku) {
   constexpr int kCT = Lay<CW>::kCT, kCW = CW;
+  Geo g = g0;
+  if (d_kl != nullptr) {
+    // enqueued by the device-side dispatch before the bandwidths were known: the
+    // decision (flags[1], set by the kernel before this one) and (kl, ku) are read
+    // here, by every CTA alike, so either all of them work or all leave now
+    if (*(volatile const int *)(flags + 1) == 0) return;
+    g.kl = *d_kl;
+    g.ku = *d_ku;
+    g.kv = g.kl + g.ku;
+  }
   extern __shared__ __align__(16) double smem[];
   __shared__ PairShared<CW> ps;
   WideShared<CW, 1> &sh = ps.w;
@@ -1035,34 +1048,80 @@ __global__ void __launch_bounds__(32 * (CW + 1), 1)
 }
 
 template <int CW>
-int launch_pair(const Geo &g, int grid, size_t smem, double *AB, int *ipiv, int *d_info, int *flags, cudaStream_t s) {
-  constexpr int kThreads = 32 * (CW + 1);
-  if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_wide_pair<CW>), 200 * 1024)) return BANDLU_ERR_CUDA;
+struct PairLaunch {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
   cudaLaunchAttribute at[2];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = 2;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  at[1].id = cudaLaunchAttributeCooperative;
-  at[1].val.cooperative = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  int clusters = 0;
-  if (cudaOccupancyMaxActiveClusters(&clusters, k_gbtrf_wide_pair<CW>, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    return BANDLU_NOT_BANDED;
+  // BANDLU_OK: the grid can be made resident (all clusters at once); BANDLU_NOT_BANDED:
+  // it cannot (the caller takes another kernel); BANDLU_ERR_CUDA.  The occupancy answer
+  // is cached per (device, grid, shared memory), so a call made during stream capture
+  // after a first call outside it issues no query.
+  int prepare(int grid, size_t smem, cudaStream_t s) {
+    if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_wide_pair<CW>), 200 * 1024))
+      return BANDLU_ERR_CUDA;
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(32 * (CW + 1));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeCooperative;
+    at[1].val.cooperative = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return BANDLU_ERR_CUDA;
+    static std::mutex mu;
+    static std::map<std::tuple<int, int, size_t>, int> fits;
+    const auto key = std::make_tuple(dev, grid, smem);
+    {
+      std::lock_guard<std::mutex> lock(mu);
+      const auto it = fits.find(key);
+      if (it != fits.end()) return it->second;
+    }
+    int clusters = 0;
+    int rc = BANDLU_OK;
+    if (cudaOccupancyMaxActiveClusters(&clusters, k_gbtrf_wide_pair<CW>, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      rc = BANDLU_NOT_BANDED;
+    } else if (clusters * 2 < grid) {
+      rc = BANDLU_NOT_BANDED;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    fits[key] = rc;
+    return rc;
   }
-  if (clusters * 2 < grid) return BANDLU_NOT_BANDED;
-  cfg.numAttrs = 2;
-  Geo gg = g;
-  if (cudaLaunchKernelEx(&cfg, k_gbtrf_wide_pair<CW>, gg, AB, ipiv, d_info, flags) != cudaSuccess)
-    return BANDLU_ERR_CUDA;
-  return BANDLU_OK;
+  int launch(const Geo &g, double *AB, int *ipiv, int *d_info, int *flags, const int *d_kl, const int *d_ku) {
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    Geo gg = g;
+    if (cudaLaunchKernelEx(&cfg, k_gbtrf_wide_pair<CW>, gg, AB, ipiv, d_info, flags, d_kl, d_ku) != cudaSuccess)
+      return BANDLU_ERR_CUDA;
+    return BANDLU_OK;
+  }
+};
+
+template <int CW>
+int launch_pair(const Geo &g, int grid, size_t smem, double *AB, int *ipiv, int *d_info, int *flags, cudaStream_t s) {
+  PairLaunch<CW> pl;
+  const int rc = pl.prepare(grid, smem, s);
+  if (rc != BANDLU_OK) return rc;
+  return pl.launch(g, AB, ipiv, d_info, flags, nullptr, nullptr);
+}
+
+template <int CW>
+int pair_fits(int grid, size_t smem, cudaStream_t s) {
+  PairLaunch<CW> pl;
+  return pl.prepare(grid, smem, s);
+}
+
+// Shared memory of the pair kernel for band storage ldab and (largest) kl.
+size_t pair_smem(long long ldab, long long kl) {
+  const size_t need_a = (size_t)kPanelBufs * kNB * (size_t)ldab + (size_t)kRB * kNB * (size_t)kl;
+  const size_t need_b = (size_t)kBBufs * kNB * (size_t)ldab;
+  const size_t need_u = (size_t)kMaxActive * kNB * (size_t)ldab;
+  return std::max(need_a, std::max(need_b, need_u)) * sizeof(double);
 }
 
 // BANDLU_WIDE_SINGLE=1 in the environment selects the single-CTA panel kernel
@@ -1140,10 +1199,7 @@ int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *
   if (rpt == 1 && sms >= 4 && !pair_disabled()) {
     // the cluster pair: CTA 0 factors, CTA 1 runs the second lookahead group
     const int grid2 = sms & ~1;
-    const size_t need_a = (size_t)kPanelBufs * kNB * (size_t)ldab + (size_t)kRB * kNB * kl;
-    const size_t need_b = (size_t)kBBufs * kNB * (size_t)ldab;
-    const size_t need_u = (size_t)kMaxActive * kNB * (size_t)ldab;
-    const size_t smem2 = std::max(need_a, std::max(need_b, need_u)) * sizeof(double);
+    const size_t smem2 = pair_smem(ldab, kl);
     if (smem2 <= 200 * 1024 && span <= (long long)kMaxActive * (grid2 - 2)) {
       if (cw == 2)
         rc = launch_pair<2>(g, grid2, smem2, AB, ipiv, d_info, flags, s);
@@ -1170,6 +1226,67 @@ int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *
   if (rc != BANDLU_OK) return rc;
   *used = true;
   return BANDLU_OK;
+}
+
+int prepare_gbtrf_wide_deferred(int64_t n, int64_t ldab, cudaStream_t s, WideDeferred *wd) {
+  *wd = WideDeferred();
+  if (pair_disabled() || n < 4 * kNB || n > INT_MAX / 2 || ldab > INT_MAX / kNB) return BANDLU_OK;
+  // the compute group is sized for the largest kl the storage admits (up to 9 warps;
+  // bands wider than the group keep the single-CTA fallback of the on-device kernel)
+  const long long kl_max = (ldab - 1) / 2;
+  const long long rows_max = kl_max + kNB;
+  const int cw = rows_max <= 64 ? 2 : (rows_max <= 128 ? 4 : 9);
+  const long long kl_cap = std::min(kl_max, (long long)32 * cw - kNB);
+  int dev = 0, sms = 0, coop = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (!coop || sms < 4) return BANDLU_OK;
+  const int grid = sms & ~1;
+  const long long span_max = (ldab - 1 + 3) / kNB + 1;  // kv <= ldab - 1
+  if (span_max > (long long)kMaxActive * (grid - 2)) return BANDLU_OK;
+  const size_t smem = pair_smem(ldab, kl_cap);
+  if (smem > 200 * 1024) return BANDLU_OK;
+  const int fit = cw == 2 ? pair_fits<2>(grid, smem, s) : (cw == 4 ? pair_fits<4>(grid, smem, s) : pair_fits<9>(grid, smem, s));
+  if (fit == BANDLU_NOT_BANDED) return BANDLU_OK;
+  if (fit != BANDLU_OK) return fit;
+  const long long npan = (n + kNB - 1) / kNB;
+  const size_t fbytes = (size_t)(2 + 2 * npan) * sizeof(int);
+  int *flags = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&flags), fbytes, s) != cudaSuccess) return BANDLU_ERR_CUDA;
+  if (cudaMemsetAsync(flags, 0, fbytes, s) != cudaSuccess) {
+    cudaFreeAsync(flags, s);
+    return BANDLU_ERR_CUDA;
+  }
+  wd->rows_cap = 32 * cw;
+  wd->cw = cw;
+  wd->grid = grid;
+  wd->smem = smem;
+  wd->flags = flags;
+  return BANDLU_OK;
+}
+
+int launch_gbtrf_wide_deferred(const WideDeferred &wd, int64_t n, double *AB, int64_t ldab, int *ipiv,
+                               const int *d_kl, const int *d_ku, int *d_info, cudaStream_t s) {
+  Geo g;
+  g.n = (int)n;
+  g.kl = g.ku = g.kv = 0;  // read on the device
+  g.ldab = ldab;
+  g.npan = (int)((n + kNB - 1) / kNB);
+  g.vec = (reinterpret_cast<uintptr_t>(AB) & 15u) == 0;
+  int rc = BANDLU_ERR_CUDA;
+  if (wd.cw == 2) {
+    PairLaunch<2> pl;
+    if (pl.prepare(wd.grid, wd.smem, s) == BANDLU_OK) rc = pl.launch(g, AB, ipiv, d_info, wd.flags, d_kl, d_ku);
+  } else if (wd.cw == 4) {
+    PairLaunch<4> pl;
+    if (pl.prepare(wd.grid, wd.smem, s) == BANDLU_OK) rc = pl.launch(g, AB, ipiv, d_info, wd.flags, d_kl, d_ku);
+  } else {
+    PairLaunch<9> pl;
+    if (pl.prepare(wd.grid, wd.smem, s) == BANDLU_OK) rc = pl.launch(g, AB, ipiv, d_info, wd.flags, d_kl, d_ku);
+  }
+  if (cudaFreeAsync(wd.flags, s) != cudaSuccess && rc == BANDLU_OK) rc = BANDLU_ERR_CUDA;
+  return rc;
 }
 
 }  // namespace bandlu

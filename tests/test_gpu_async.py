@@ -101,3 +101,54 @@ def test_dispatch_lu_async_in_a_cuda_graph():
         g.replay()
         torch.cuda.synchronize()
         check_against_oracle(A, ldab, out)
+
+
+@pytest.mark.parametrize("n,kl,ku,ldab", [(2049, 256, 256, 769), (1200, 40, 30, 111), (3000, 100, 20, 221)])
+def test_dispatch_lu_async_wide_bands(n, kl, ku, ldab):
+    """Wide bands: the multi-CTA cluster kernel, enqueued before the bandwidths are known, takes
+    them on the device; bit-identical to dispatch_lu (which chose the same kernel on the host)
+    and to the oracle."""
+    A = make_dense(n, kl, ku, dist="uniform", diag_boost=0.0, seed=n + 7 * kl).numpy()
+    out = AsyncOut(n, ldab)
+    Ad = torch.from_numpy(A).to(DEV)
+    assert out.call(Ad, n, n, ldab) == 0
+    AB = torch.zeros((n, ldab), dtype=torch.float64, device=DEV)
+    ipiv = torch.zeros(n, dtype=torch.int32, device=DEV)
+    info = torch.zeros(1, dtype=torch.int32, device=DEV)
+    rc, gkl, gku = bandlu.dispatch_lu(Ad, n, n, AB, ldab, ipiv, info)
+    torch.cuda.synchronize()
+    kl2, ku2, status, info2, AB2, ipiv2 = out.result()
+    assert (rc, gkl, gku, int(info.item())) == (status, kl2, ku2, info2) == (0, kl, ku, 0)
+    assert np.array_equal(AB.cpu().numpy().view(np.int64), AB2.view(np.int64))
+    assert torch.equal(ipiv.cpu(), torch.from_numpy(ipiv2))
+    check_against_oracle(A, ldab, out)
+
+
+def test_dispatch_lu_async_wide_band_in_a_cuda_graph():
+    """One capture with band storage that admits wide bands, replayed on a wide band (the
+    multi-CTA kernel), a narrow one (register window), a windowed one and a declined one."""
+    n, ldab = 1500, 121
+    mats = [make_dense(n, 40, 30, dist="uniform", diag_boost=0.0, seed=21).numpy(),
+            make_dense(n, 3, 3, dist="uniform", diag_boost=0.0, seed=22).numpy(),
+            make_dense(n, 20, 50, dist="uniform", diag_boost=0.0, seed=23).numpy(),
+            make_dense(n, 50, 20, dist="uniform", diag_boost=0.0, seed=24).numpy()]
+    mats[3][n - 1, 0] = 1e-3  # declined: kl = n-1
+    Ad = torch.zeros((n, n), dtype=torch.float64, device=DEV)
+    out = AsyncOut(n, ldab)
+    s = torch.cuda.Stream()
+    Ad.copy_(torch.from_numpy(mats[0]))
+    with torch.cuda.stream(s):
+        assert out.call(Ad, n, n, ldab) == 0  # warm-up outside the capture
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        rc = out.call(Ad, n, n, ldab)
+    assert rc == 0
+    for A in mats:
+        out.AB.fill_(-3.0)
+        out.ipiv.fill_(-1)
+        out.sc.fill_(-7)
+        Ad.copy_(torch.from_numpy(A))
+        g.replay()
+        torch.cuda.synchronize()
+        check_against_oracle(A, ldab, out)
