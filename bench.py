@@ -370,6 +370,19 @@ def run_peaks(args):
             bandlu.bandlu_peak_hbm_read(buf, nbytes, sink, blocks, stream), "hbm_read"), 5)
         rd[f"blocks{blocks}"] = nbytes / (min(ts) * 1e-3) / 1e9
     out["hbm_read_gbs_4gib"] = rd
+    # the same read-only stream over 128 MiB (the size of the n = 4096 dense matrix), L2 flushed
+    # before each read: the ceiling a detection pass of that size can reach (ramp and tail included)
+    flush = L2Flush(torch, dev)
+    small = {}
+    for nbytes_s in (128 << 20, 512 << 20):
+        for bps in (2, 4):
+            blocks = sms * bps
+            sink = torch.empty(blocks, dtype=torch.int64, device=dev)
+            ts = event_ms(torch, stream, lambda: bandlu.check(
+                bandlu.bandlu_peak_hbm_read(buf, nbytes_s, sink, blocks, stream), "hbm_read"), 10, flush)
+            small[f"{nbytes_s >> 20}MiB_blocks{blocks}"] = {"us": statistics.median(ts) * 1e3,
+                                                            "gbs": nbytes_s / (statistics.median(ts) * 1e-3) / 1e9}
+    out["hbm_read_cold"] = small
     # clock while the FMA kernel runs, for the per-clock rates
     sampler = ClockSampler(0)
     sampler.start()
@@ -395,6 +408,19 @@ def run_peaks(args):
 
 # ---------------------------------------------------------------------------------------
 # the per-workload measurements beside the contract line
+
+def plain_read_s(torch, bandlu, A, dev, stream, flush, reps: int):
+    """Median time of one read-only pass (bandlu_peak_hbm_read) over the same dense matrix,
+    L2 flushed before each: the ceiling a detection pass over those bytes can reach."""
+    nbytes = A.numel() * 8
+    if nbytes < 16 or nbytes % 16 or A.data_ptr() % 16:
+        return None
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    sink = torch.empty(4 * sms, dtype=torch.int64, device=dev)
+    ts = event_ms(torch, stream, lambda: bandlu.check(
+        bandlu.bandlu_peak_hbm_read(A, nbytes, sink, 4 * sms, stream), "hbm_read"), reps, flush)
+    return statistics.median(ts) * 1e-3
+
 
 def measure_single(torch, bandlu, w, dev, stream, flush, reps: int, fp64_peak: float, hbm_peak: float,
                    dense_ms=None):
@@ -431,8 +457,10 @@ def measure_single(torch, bandlu, w, dev, stream, flush, reps: int, fp64_peak: f
         raise RuntimeError(f"{w.name}: dispatch_lu_async disagrees with dispatch_lu")
     del ABa, ipa
     det_bytes = 8.0 * n * n
+    t_read = plain_read_s(torch, bandlu, A, dev, stream, flush, reps)
     out = {"status": rc, "detected_kl": dkl, "detected_ku": dku, "dispatch_ms": t_disp * 1e3,
-           "dispatch_async_ms": t_async * 1e3,
+           "dispatch_async_ms": t_async * 1e3, "plain_read_us": t_read * 1e6 if t_read else None,
+           "detect_frac_of_plain_read": (t_read / t_det) if t_read else None,
            "detect_us": t_det * 1e6, "detect_gbs": det_bytes / t_det / 1e9,
            "detect_frac_hbm": det_bytes / t_det / 1e9 / hbm_peak}
     if rc == 0:
@@ -602,12 +630,14 @@ def run_ours(args):
     barrier()
     torch.cuda.synchronize()
     t_wall0 = time.time()
+    torch.cuda.nvtx.range_push("timed_steps")  # lets a profiler select exactly these launches
     for k in range(args.steps):
         flush(k)                       # L2 flush between steps, outside the timed events
         starts[k].record(stream)
         step()
         ends[k].record(stream)
     torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
     barrier()
     t_wall1 = time.time()
     if rank == 0:
@@ -660,9 +690,12 @@ def run_ours(args):
     convert_bytes = 8.0 * nnz_band + 8.0 * ldab * n
     band_bytes = 2 * 8.0 * ldab * n
     fac_kernel = gbtrf_kernel(n, kl, ku)
+    t_read = plain_read_s(torch, bandlu, A, dev, stream, flush, reps)
     stages = {
         "detect_us": t_detect * 1e6, "detect_gbs": detect_bytes / t_detect / 1e9,
         "detect_frac_hbm": detect_bytes / t_detect / 1e9 / hbm_peak,
+        "plain_read_us": t_read * 1e6 if t_read else None,
+        "detect_frac_of_plain_read": (t_read / t_detect) if t_read else None,
         "convert_us": t_convert * 1e6, "convert_gbs": convert_bytes / t_convert / 1e9,
         "gbtrf_kernel": fac_kernel, "gbtrf_us": t_gbtrf * 1e6, "gbtrf_gflops": flops / t_gbtrf / 1e9,
         "gbtrf_ns_per_column": t_gbtrf / n * 1e9, "gbtrf_frac_fp64": flops / t_gbtrf / 1e9 / fp64_peak,
