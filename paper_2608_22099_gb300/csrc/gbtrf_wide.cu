@@ -864,9 +864,12 @@ __global__ void __launch_bounds__(32 * (CW + 1), 1)
       if (g.npan > 1) load_block(g, AB, buf(1), 1, true, tid, kCT);
       bar_compute<CW>();
       for (int p = 0; p < g.npan; ++p) {
-        // ring entry p % kRB last held panel p - kRB, which CTA 1 reads: wait until it has
+        // ring entry p % kRB last held panel p - kRB, which CTA 1 reads: wait until it has.
+        // Only a write-after-read order is needed: CTA 1's loads of the entry are performed
+        // before its arrival (they precede a barrier and a release), and this CTA writes the
+        // entry only after observing that arrival, so a CTA-scope poll suffices here.
         if (p >= kRB && p - kRB + 2 < g.npan &&
-            !grp_wait_cl(&ps.mb_credit[p % kRB], ring_parity(p - kRB, kRB), kBarA))
+            !grp_wait_local(&ps.mb_credit[p % kRB], ring_parity(p - kRB, kRB), kBarA))
           break;
         factor_panel<CW, 1>(g, buf(p), p, mults(p), sh, bpar, info);
         if (tid == 0) {
