@@ -390,6 +390,23 @@ def run_peaks(args):
             small[f"{nbytes_s >> 20}MiB_blocks{blocks}"] = {"us": statistics.median(ts) * 1e3,
                                                             "gbs": nbytes_s / (statistics.median(ts) * 1e-3) / 1e9}
     out["hbm_read_cold"] = small
+    # per-warp cost of the operations a column step is made of, in SM clocks, on one block of
+    # 1, 3 and 4 warps (include/bandlu_peaks.h): what the latency-bound factorisations pay
+    ops = ("dfma_dependent", "dfma_independent", "shfl_f64_dependent", "shfl_b32_independent",
+           "smem_roundtrip", "imad_dependent", "redux_ballot_dependent", "rcp_rn_dependent")
+    clk_buf = torch.zeros(1, dtype=torch.int64, device=dev)
+    sink_w = torch.empty(32 * 32, dtype=torch.float64, device=dev)
+    costs = {}
+    for op, name in enumerate(ops):
+        row = {}
+        for warps in (1, 3, 4):
+            iters = 256
+            for _ in range(2):  # the second launch is the measured one
+                bandlu.check(bandlu.bandlu_peak_warp_costs(op, clk_buf, sink_w, warps, iters, stream), "warp_costs")
+            torch.cuda.synchronize()
+            row[f"warps{warps}"] = round(int(clk_buf.item()) / (16 * iters), 1)
+        costs[name] = row
+    out["warp_costs_clk"] = costs
     # clock while the FMA kernel runs, for the per-clock rates
     sampler = ClockSampler(0)
     sampler.start()

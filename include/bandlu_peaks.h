@@ -46,6 +46,23 @@ int bandlu_peak_dmma(int shape, double *d_sink, int blocks, int warps, int chain
 int bandlu_peak_hbm_read(const void *d_buf, int64_t bytes, unsigned long long *d_sink, int blocks,
                          cudaStream_t stream);
 
+/* Per-warp cost of one operation, in SM clock cycles.  ONE block of `warps` warps
+ * (1..32) runs `iters` (>= 1) rounds of 16 instances of operation `op`:
+ *   0  dependent fma(a, b, c) in FP64 (each uses the previous result)
+ *   1  independent FP64 fma (8 chains per thread, two rounds)
+ *   2  dependent 64-bit warp shuffle of a double (__shfl_sync, source lane + 1)
+ *   3  independent 32-bit warp shuffles
+ *   4  shared-memory round trip: a store, __syncwarp, a load of a neighbour's value
+ *   5  dependent 32-bit integer multiply-add
+ *   6  dependent redux.sync max + ballot (the pivot search's reduction)
+ *   7  dependent correctly rounded FP64 reciprocal (the library's integer-pipe
+ *      reciprocal of Sec. III-A's multipliers, x -> 1/x)
+ * d_clk: 1 word, thread 0's clock64 cycles over the rounds (cycles per operation
+ * per warp = *d_clk / (16 * iters)); d_sink: 32 * warps doubles (keeps the
+ * results live).  op outside 0..7 is argument 1. */
+int bandlu_peak_warp_costs(int op, unsigned long long *d_clk, double *d_sink, int warps, int iters,
+                           cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

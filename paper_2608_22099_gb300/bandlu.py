@@ -83,7 +83,8 @@ def load():
         lib.bandlu_peak_dfma.argtypes = [vp, i32, i32, i32, i32, vp]
         lib.bandlu_peak_dmma.argtypes = [i32, vp, i32, i32, i32, i32, vp]
         lib.bandlu_peak_hbm_read.argtypes = [vp, i64, vp, i32, vp]
-        for f in ("bandlu_peak_dfma", "bandlu_peak_dmma", "bandlu_peak_hbm_read"):
+        lib.bandlu_peak_warp_costs.argtypes = [i32, vp, vp, i32, i32, vp]
+        for f in ("bandlu_peak_dfma", "bandlu_peak_dmma", "bandlu_peak_hbm_read", "bandlu_peak_warp_costs"):
             getattr(lib, f).restype = ctypes.c_int
         lib.bandlu_version.restype = ctypes.c_char_p
         lib.bandlu_version.argtypes = []
@@ -240,6 +241,12 @@ def bandlu_peak_dfma(d_sink, blocks: int, threads: int, chains: int, iters: int,
 def bandlu_peak_dmma(shape: int, d_sink, blocks: int, warps: int, chains: int, iters: int, stream=None) -> int:
     """Microbenchmark launch: FP64 mma.sync (shape 0 m8n8k4, 1 m16n8k16), chains accumulators per warp."""
     return load().bandlu_peak_dmma(shape, _ptr(d_sink), blocks, warps, chains, iters, _stream(stream))
+
+
+def bandlu_peak_warp_costs(op: int, d_clk, d_sink, warps: int, iters: int, stream=None) -> int:
+    """Microbenchmark launch: one block of `warps` warps, 16 * iters instances of operation `op`
+    (0..7, see include/bandlu_peaks.h); d_clk receives thread 0's elapsed clock cycles."""
+    return load().bandlu_peak_warp_costs(op, _ptr(d_clk), _ptr(d_sink), warps, iters, _stream(stream))
 
 
 def bandlu_peak_hbm_read(d_buf, nbytes: int, d_sink, blocks: int, stream=None) -> int:

@@ -6,6 +6,7 @@
 // GB300 delivers for each, so the benchmark's fractions use measured ceilings.
 #include "bandlu_peaks.h"
 #include "common.cuh"
+#include "rcp.cuh"
 
 namespace {
 
@@ -112,6 +113,69 @@ __global__ void __launch_bounds__(512) k_peak_read(const ulonglong2 *__restrict_
   if (threadIdx.x == 0) sink[blockIdx.x] = acc;
 }
 
+// One block; thread 0 times `iters` rounds of 16 instances of one operation.
+template <int OP>
+__global__ void k_peak_warp_costs(unsigned long long *__restrict__ clk, double *__restrict__ sink, int iters) {
+  __shared__ __align__(16) double sm[32][32];
+  const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+  double x = 1.0 + 1e-3 * lane, c8[8];
+  unsigned u = 7u * lane + 3u;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) c8[k] = x + k;
+  sm[w][lane] = x;
+  __syncthreads();
+  const long long t0 = clock64();
+  for (int it = 0; it < iters; ++it) {
+    if constexpr (OP == 0) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) x = fma(x, 0.9999999999999, 1e-12);
+    } else if constexpr (OP == 1) {
+#pragma unroll
+      for (int r = 0; r < 2; ++r)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) c8[k] = fma(c8[k], 0.9999999999999, 1e-12);
+    } else if constexpr (OP == 2) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) x = __shfl_sync(bandlu::FULL, x, (lane + 1) & 31);
+    } else if constexpr (OP == 3) {
+      unsigned a = 0u;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) a += __shfl_sync(bandlu::FULL, u, (lane + j) & 31);
+      u += a & 1u;
+    } else if constexpr (OP == 4) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        sm[w][lane] = x;
+        __syncwarp();
+        x = ((volatile double *)sm[w])[(lane + 1) & 31];
+        __syncwarp();
+      }
+    } else if constexpr (OP == 5) {
+      // opaque to the compiler, which would otherwise fold the affine recurrence
+#pragma unroll
+      for (int j = 0; j < 16; ++j) asm volatile("mad.lo.u32 %0, %0, %1, %2;" : "+r"(u) : "r"(2654435761u), "r"(lane));
+    } else if constexpr (OP == 6) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const unsigned m = __reduce_max_sync(bandlu::FULL, u);
+        u += (__ballot_sync(bandlu::FULL, u == m) & 1u) + 1u;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        bool special;
+        x = bandlu::rcp_rn_fast(x, &special);
+      }
+    }
+  }
+  const long long t1 = clock64();
+  double s = x + (double)u;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) s += c8[k];
+  sink[t] = s;
+  if (t == 0) *clk = (unsigned long long)(t1 - t0);
+}
+
 }  // namespace
 
 extern "C" {
@@ -170,6 +234,28 @@ int bandlu_peak_hbm_read(const void *d_buf, int64_t bytes, unsigned long long *d
   if (d_sink == nullptr) return -3;
   if (blocks < 1) return -4;
   k_peak_read<<<blocks, 512, 0, stream>>>(static_cast<const ulonglong2 *>(d_buf), bytes / 16, d_sink);
+  BANDLU_CHECK_LAUNCH();
+  return BANDLU_OK;
+}
+
+int bandlu_peak_warp_costs(int op, unsigned long long *d_clk, double *d_sink, int warps, int iters,
+                           cudaStream_t stream) {
+  if (op < 0 || op > 7) return -1;
+  if (d_clk == nullptr) return -2;
+  if (d_sink == nullptr) return -3;
+  if (warps < 1 || warps > 32) return -4;
+  if (iters < 1) return -5;
+  const int t = 32 * warps;
+  switch (op) {
+    case 0: k_peak_warp_costs<0><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+    case 1: k_peak_warp_costs<1><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+    case 2: k_peak_warp_costs<2><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+    case 3: k_peak_warp_costs<3><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+    case 4: k_peak_warp_costs<4><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+    case 5: k_peak_warp_costs<5><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+    case 6: k_peak_warp_costs<6><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+    default: k_peak_warp_costs<7><<<1, t, 0, stream>>>(d_clk, d_sink, iters); break;
+  }
   BANDLU_CHECK_LAUNCH();
   return BANDLU_OK;
 }

@@ -276,3 +276,21 @@ BIG = 1 << 62  # a leading dimension or stride whose extent over the matrix woul
 ])
 def test_overflowing_extents_are_rejected(call, expect):
     assert call() == expect
+
+
+def test_peak_microbenchmarks_reject_bad_arguments():
+    # the argument checks run on the host before any launch (stream 0: no CUDA call)
+    assert bandlu.bandlu_peak_warp_costs(8, DEV, DEV, 1, 1, 0) == -1
+    assert bandlu.bandlu_peak_warp_costs(-1, DEV, DEV, 1, 1, 0) == -1
+    assert bandlu.bandlu_peak_warp_costs(0, 0, DEV, 1, 1, 0) == -2
+    assert bandlu.bandlu_peak_warp_costs(0, DEV, 0, 1, 1, 0) == -3
+    assert bandlu.bandlu_peak_warp_costs(0, DEV, DEV, 0, 1, 0) == -4
+    assert bandlu.bandlu_peak_warp_costs(0, DEV, DEV, 33, 1, 0) == -4
+    assert bandlu.bandlu_peak_warp_costs(0, DEV, DEV, 1, 0, 0) == -5
+    assert bandlu.bandlu_peak_dfma(0, 1, 32, 1, 1, 0) == -1
+    assert bandlu.bandlu_peak_dfma(DEV, 1, 48, 1, 1, 0) == -3
+    assert bandlu.bandlu_peak_dfma(DEV, 1, 32, 9, 1, 0) == -4
+    assert bandlu.bandlu_peak_dmma(2, DEV, 1, 1, 1, 1, 0) == -1
+    assert bandlu.bandlu_peak_dmma(0, DEV, 1, 1, 5, 1, 0) == -5
+    assert bandlu.bandlu_peak_hbm_read(DEV + 8, 64, DEV, 1, 0) == -1
+    assert bandlu.bandlu_peak_hbm_read(DEV, 24, DEV, 1, 0) == -2

@@ -500,7 +500,10 @@ def test_batched_many_small_varied_bands():
 
 
 @pytest.mark.parametrize("batch,n,kl,ku,lda", [(37, 256, 2, 2, 256), (16, 100, 3, 1, 101), (8, 1, 0, 0, 1),
-                                               (5, 700, 10, 10, 700)])
+                                               (5, 700, 10, 10, 700),
+                                               # column windows: kl = 7 in 8 row registers (ldab 16),
+                                               # and 8 matrices per warp (ldab 3)
+                                               (12, 50, 7, 1, 50), (33, 64, 1, 0, 64)])
 def test_batched_matches_oracle(batch, n, kl, ku, lda):
     A = make_dense(n, kl, ku, dist="uniform", diag_boost=0.0, seed=batch + n, batch=batch, lda=lda)
     ldab = 2 * kl + ku + 1
