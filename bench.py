@@ -55,7 +55,8 @@ FALLBACK_HBM_GBS = 6800.0
 # Sources of each kernel: a DRAM-traffic figure taken by ncu is valid only while
 # their hash is the one recorded beside it under profiles/.
 KERNEL_SOURCES = {
-    "k_gbtrf_wide": ["gbtrf_wide.cu", "common.cuh", "rcp.cuh", "sync.cuh"],
+    "k_gbtrf_wide": ["gbtrf_wide.cu", "gbtrf_wide_stream.cuh", "common.cuh", "rcp.cuh", "sync.cuh"],
+    "k_gbtrf_wide_chain": ["gbtrf_wide.cu", "gbtrf_wide_stream.cuh", "common.cuh", "rcp.cuh", "sync.cuh"],
     "k_gbtrf_window": ["gbtrf.cu", "common.cuh", "rcp.cuh", "sync.cuh", "regwin.cuh"],
     "k_gbtrf_regwin": ["gbtrf.cu", "common.cuh", "rcp.cuh", "sync.cuh", "regwin.cuh"],
     "k_detect_vec": ["detect.cu", "common.cuh"],
@@ -102,6 +103,9 @@ def gbtrf_kernel(n: int, kl: int, ku: int) -> str:
         return "k_gbtrf_regwin"
     if kl <= 27:
         return "k_gbtrf_window"
+    if (kl + 4 <= 288 and kl + ku >= 8 and n >= 16 and os.environ.get("BANDLU_WIDE_SINGLE") != "1"
+            and os.environ.get("BANDLU_WIDE_PAIR") != "1"):
+        return "k_gbtrf_wide_chain"  # where its clusters of five fit (else the pair or single-CTA kernel)
     return "k_gbtrf_wide"
 
 

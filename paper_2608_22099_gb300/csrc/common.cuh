@@ -158,6 +158,7 @@ int launch_gbtrf_on_device(int64_t n, double *AB, int64_t ldab, int *ipiv, const
 struct WideDeferred {
   int rows_cap = 0;
   int cw = 0;
+  bool chain = false;  // the streaming chain kernel (else the cluster pair)
   int grid = 0;
   size_t smem = 0;
   int *flags = nullptr;

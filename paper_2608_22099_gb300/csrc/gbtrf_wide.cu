@@ -1,6 +1,15 @@
 // gbtrf_wide.cu -- banded LU for wide bands (kl beyond the windowed kernel):
-// a persistent, cooperatively launched kernel, one CTA per SM (Sec. II-A step 3;
-// f(N) ~ O(N*P*Q), Eq. S-N-N3).
+// persistent, cooperatively launched kernels, one CTA per SM (Sec. II-A step 3;
+// f(N) ~ O(N*P*Q), Eq. S-N-N3).  Three variants share the step functions below:
+//
+//  * k_gbtrf_wide_chain (gbtrf_wide_stream.cuh), the default when a panel row
+//    fits one thread: CTA 0 only factors, and the lookahead panels stream down a
+//    cluster of streaming CTAs;
+//  * k_gbtrf_wide_pair, when the chain's clusters cannot all be resident: CTA 0
+//    factors and looks ahead, a second lookahead group runs on its cluster
+//    partner;
+//  * k_gbtrf_wide (described first, below), the single panel CTA, for up to four
+//    rows per thread and wherever no cluster kernel fits.
 //
 // Columns are cut into blocks of kNB; block p is panel p.
 //
@@ -1127,6 +1136,8 @@ size_t pair_smem(long long ldab, long long kl) {
   return std::max(need_a, std::max(need_b, need_u)) * sizeof(double);
 }
 
+#include "gbtrf_wide_stream.cuh"
+
 // BANDLU_WIDE_SINGLE=1 in the environment selects the single-CTA panel kernel
 // for every shape (read once): the comparison the cluster pair is measured against.
 bool pair_disabled() {
@@ -1200,10 +1211,32 @@ int launch_gbtrf_wide(int64_t n, int kl, int ku, double *AB, int64_t ldab, int *
   }
   int rc = BANDLU_NOT_BANDED;
   if (rpt == 1 && sms >= 4 && !pair_disabled()) {
-    // the cluster pair: CTA 0 factors, CTA 1 runs the second lookahead group
+    if (!chain_disabled()) {
+      // the chain: CTA 0 factors, kStreamers CTAs apply the lookahead panels as they stream in
+      const size_t smemc = stream_smem(ldab, cw);
+      if (smemc <= 200 * 1024) {
+        auto run = [&](auto &sl) {
+          const int gc = sl.prepare(sms, smemc, s);
+          if (gc < 0) return BANDLU_ERR_CUDA;
+          if (gc == 0 || span > (long long)kMaxActive * (gc - kChainCTAs)) return BANDLU_NOT_BANDED;
+          return sl.launch(g, AB, ipiv, d_info, flags, nullptr, nullptr);
+        };
+        if (cw == 2) {
+          StreamLaunch<2> sl;
+          rc = run(sl);
+        } else if (cw == 4) {
+          StreamLaunch<4> sl;
+          rc = run(sl);
+        } else {
+          StreamLaunch<9> sl;
+          rc = run(sl);
+        }
+      }
+    }
+    // the cluster pair: CTA 0 factors and looks ahead, CTA 1 runs the second lookahead group
     const int grid2 = sms & ~1;
     const size_t smem2 = pair_smem(ldab, kl);
-    if (smem2 <= 200 * 1024 && span <= (long long)kMaxActive * (grid2 - 2)) {
+    if (rc == BANDLU_NOT_BANDED && smem2 <= 200 * 1024 && span <= (long long)kMaxActive * (grid2 - 2)) {
       if (cw == 2)
         rc = launch_pair<2>(g, grid2, smem2, AB, ipiv, d_info, flags, s);
       else if (cw == 4)
@@ -1245,14 +1278,41 @@ int prepare_gbtrf_wide_deferred(int64_t n, int64_t ldab, cudaStream_t s, WideDef
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
   if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) return BANDLU_ERR_CUDA;
   if (!coop || sms < 4) return BANDLU_OK;
-  const int grid = sms & ~1;
   const long long span_max = (ldab - 1 + 3) / kNB + 1;  // kv <= ldab - 1
-  if (span_max > (long long)kMaxActive * (grid - 2)) return BANDLU_OK;
-  const size_t smem = pair_smem(ldab, kl_cap);
-  if (smem > 200 * 1024) return BANDLU_OK;
-  const int fit = cw == 2 ? pair_fits<2>(grid, smem, s) : (cw == 4 ? pair_fits<4>(grid, smem, s) : pair_fits<9>(grid, smem, s));
-  if (fit == BANDLU_NOT_BANDED) return BANDLU_OK;
-  if (fit != BANDLU_OK) return fit;
+  int grid = 0;
+  size_t smem = 0;
+  bool chain = false;
+  if (!chain_disabled() && stream_smem(ldab, cw) <= 200 * 1024) {
+    // the chain, as in launch_gbtrf_wide
+    const size_t smemc = stream_smem(ldab, cw);
+    int gc = 0;
+    if (cw == 2) {
+      StreamLaunch<2> sl;
+      gc = sl.prepare(sms, smemc, s);
+    } else if (cw == 4) {
+      StreamLaunch<4> sl;
+      gc = sl.prepare(sms, smemc, s);
+    } else {
+      StreamLaunch<9> sl;
+      gc = sl.prepare(sms, smemc, s);
+    }
+    if (gc < 0) return BANDLU_ERR_CUDA;
+    if (gc > 0 && span_max <= (long long)kMaxActive * (gc - kChainCTAs)) {
+      chain = true;
+      grid = gc;
+      smem = smemc;
+    }
+  }
+  if (!chain) {
+    grid = sms & ~1;
+    if (span_max > (long long)kMaxActive * (grid - 2)) return BANDLU_OK;
+    smem = pair_smem(ldab, kl_cap);
+    if (smem > 200 * 1024) return BANDLU_OK;
+    const int fit =
+        cw == 2 ? pair_fits<2>(grid, smem, s) : (cw == 4 ? pair_fits<4>(grid, smem, s) : pair_fits<9>(grid, smem, s));
+    if (fit == BANDLU_NOT_BANDED) return BANDLU_OK;
+    if (fit != BANDLU_OK) return fit;
+  }
   const long long npan = (n + kNB - 1) / kNB;
   const size_t fbytes = (size_t)(2 + 2 * npan) * sizeof(int);
   int *flags = nullptr;
@@ -1263,6 +1323,7 @@ int prepare_gbtrf_wide_deferred(int64_t n, int64_t ldab, cudaStream_t s, WideDef
   }
   wd->rows_cap = 32 * cw;
   wd->cw = cw;
+  wd->chain = chain;
   wd->grid = grid;
   wd->smem = smem;
   wd->flags = flags;
@@ -1278,7 +1339,22 @@ int launch_gbtrf_wide_deferred(const WideDeferred &wd, int64_t n, double *AB, in
   g.npan = (int)((n + kNB - 1) / kNB);
   g.vec = (reinterpret_cast<uintptr_t>(AB) & 15u) == 0;
   int rc = BANDLU_ERR_CUDA;
-  if (wd.cw == 2) {
+  if (wd.chain) {
+    auto run = [&](auto &sl) {
+      return sl.prepare(device_sms(), wd.smem, s) == wd.grid ? sl.launch(g, AB, ipiv, d_info, wd.flags, d_kl, d_ku)
+                                                             : BANDLU_ERR_CUDA;
+    };
+    if (wd.cw == 2) {
+      StreamLaunch<2> sl;
+      rc = run(sl);
+    } else if (wd.cw == 4) {
+      StreamLaunch<4> sl;
+      rc = run(sl);
+    } else {
+      StreamLaunch<9> sl;
+      rc = run(sl);
+    }
+  } else if (wd.cw == 2) {
     PairLaunch<2> pl;
     if (pl.prepare(wd.grid, wd.smem, s) == BANDLU_OK) rc = pl.launch(g, AB, ipiv, d_info, wd.flags, d_kl, d_ku);
   } else if (wd.cw == 4) {

@@ -1,0 +1,672 @@
+// gbtrf_wide_stream.cuh -- the wide-band factorisation (Sec. II-A step 3; f(N) ~
+// O(N*P*Q), Eq. S-N-N3) with the lookahead taken off the panel CTA and streamed
+// down a chain of CTAs.  Included by gbtrf_wide.cu inside its anonymous
+// namespace (it uses that file's block transfers, step functions and bounded
+// waits).
+//
+// Cluster 0 holds 1 + kStreamers CTAs:
+//
+//  * CTA 0 (A) only factors: block p arrives with panels 0..p-1 applied, group A
+//    factors it, and after every column step each thread sends its row's
+//    multiplier (thread 0 also the step's pivot offset and zero flag) into the
+//    streamers' shared memory with one 8-byte st.async per streamer, completing
+//    a transaction count on that streamer's barrier of the step.  A storer warp
+//    writes finished panels to AB and publishes them.
+//  * CTA r (streamer r, 1 <= r <= kStreamers) receives every block b from CTA
+//    r+1 (streamer kStreamers from its loader, which takes the block from AB once
+//    an update CTA has applied panels p_first(b)..b-kHandChain), applies panel
+//    b-r to it as that panel's steps arrive (the pivot row and row j broadcast
+//    inside the CTA, which holds the whole block), and passes the block to CTA
+//    r-1 with one shared-to-shared bulk copy.  While A factors panel p, streamer
+//    r applies panel p to block p+r, so each block reaches A with panels up to
+//    p-1 applied, at most one step after A's last step plus one copy.
+//  * The other CTAs (update CTAs) apply panels p_first(b)..b-kHandChain and hand
+//    block b over (block_ready[b]).
+//
+// Panels are applied to a block in increasing order by whichever CTA holds it,
+// with the step functions of the other kernels, so the factors are
+// bit-identical to the unblocked elimination.  Rings without credits: the step
+// records of panel p overwrite those of panel p-kRecDepth, which every streamer
+// has read before A can hold block p (each streamer has passed block p on, after
+// reading panel p-kStreamers); a block goes into a slot whose previous block
+// (b-kSlots) A has already factored (panel_ready).  Every wait is bounded.
+#pragma once
+
+constexpr int kStreamers = 4;                    // streamer CTAs after A
+constexpr int kChainCTAs = kStreamers + 1;       // cluster size
+constexpr int kRecDepth = kStreamers + 1;        // panels of step records per streamer
+constexpr int kSlots = kStreamers + 2;           // block slots per streamer
+constexpr int kHandChain = kStreamers + 1;       // update CTAs hand block b over after panel b-kHandChain
+
+template <int CW>
+struct StreamShared {
+  WideShared<CW, 1> w;
+  unsigned long long mb_rec[kRecDepth * kNB];  // streamer: step (q, k) arrived (1 arrival + bytes), event q / kRecDepth
+  unsigned long long mb_in[kSlots];            // streamer: block b in slot (b-1) % kSlots, event (b-1) / kSlots
+  unsigned long long mb_blk[kRing];            // A: block b >= 1 arrived (1 arrival + bytes), event b-1
+  unsigned long long mb_afree[kRing];          // streamer 1: A's buffer of block p stored (A's storer), event p
+  unsigned long long mb_pub[kRing];            // A: panel p published (publisher), event p
+  alignas(16) unsigned long long rhdr[kRecDepth * kNB][2];  // streamer: pivot offset and zero flag of (q, k)
+};
+
+__device__ __forceinline__ unsigned long long dbl_bits_w(double x) {
+  return (unsigned long long)__double_as_longlong(x);
+}
+__device__ __forceinline__ void st_async_b64(unsigned raddr, unsigned long long v, unsigned rbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b64 [%0], %1, [%2];" ::"r"(raddr), "l"(v),
+               "r"(rbar)
+               : "memory");
+}
+__device__ __forceinline__ void st_async_v2(unsigned raddr, unsigned long long a, unsigned long long b,
+                                            unsigned rbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.b64 [%0], {%1, %2}, [%3];" ::"r"(raddr),
+               "l"(a), "l"(b), "r"(rbar)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx_local(unsigned long long *bar, unsigned bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes) : "memory");
+}
+
+// The group's barrier, returning true iff every thread of the group passes ok.
+template <int CW>
+__device__ __forceinline__ bool bar_and_group(int id, bool ok) {
+  unsigned r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(ok ? 1u : 0u), "r"(id), "n"(Lay<CW>::kCT)
+      : "memory");
+  return r != 0;
+}
+
+// I/O warp wait: every lane polls the same condition, so the warp never diverges
+// around the wait; the outcome is made uniform.
+template <class F>
+__device__ __forceinline__ bool io_wait_all(F ready, int *err) {
+  const bool ok = bounded_poll(ready, err);
+  return __all_sync(FULL, ok);
+}
+
+// Where the records of panel p go on each streamer (cluster addresses); bit r-1
+// of mask: streamer r consumes panel p (block p+r exists).
+struct RecTarget {
+  unsigned rec[kStreamers];  // multiplier slots of step 0 (step k: + k * kCT * 8)
+  unsigned hdr[kStreamers];  // header of step 0 (step k: + k * 16)
+  unsigned bar[kStreamers];  // barrier of step 0 (step k: + k * 8)
+  unsigned mask;
+};
+
+// factor_panel for one row per thread, streaming each step's multipliers to the streamers.
+template <int CW>
+__device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared<CW, 1> &sh, int &bpar, int &info,
+                                    const RecTarget &rt) {
+  constexpr int kCT = Lay<CW>::kCT, kCW = CW;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int c0 = p * kNB, nc = min(kNB, g.n - c0);
+  const int ldab = (int)g.ldab;
+  const int pp = p & 1;
+  const int i = tid, row = c0 + i;
+  const bool mine = i < g.kl + kNB && row < g.n;
+  double v[kNB];
+#pragma unroll
+  for (int k = 0; k < kNB; ++k) v[k] = (mine && k < nc && i - k <= g.kl) ? blk[k * ldab + g.kv + i - k] : 0.0;
+#pragma unroll
+  for (int k = 0; k < kNB; ++k) {
+    if (k >= nc) break;
+    const int j = c0 + k, km = min(g.kl, g.n - 1 - j);
+    const int s = bpar;
+    bpar ^= 1;
+    const int t = i - k;
+    bool myspec;
+    const double myr = rcp_rn_fast(v[k], &myspec);
+    const unsigned long long key = (t >= 0 && t <= km) ? pivot_key(v[k], t == 0) : 0ull;
+    unsigned long long kmax;
+    const int wl = warp_first_max(key, &kmax);
+    if (lane == wl) {
+      sh.key[s][warp] = kmax;
+      sh.idx[s][warp] = i;
+#pragma unroll
+      for (int d = 0; d < kNB; ++d) sh.piv[s][warp][d] = v[d];
+      sh.pivm[s][warp] = nz_mask(v);
+      sh.prc[s][warp] = myr;
+      sh.pspec[s][warp] = myspec ? 1 : 0;
+    }
+    if (i == k) {
+#pragma unroll
+      for (int d = 0; d < kNB; ++d) sh.row0[s][d] = v[d];
+    }
+    bar_compute<CW>();
+    int wb = 0;
+    if constexpr (kCW <= 32) {
+      const unsigned long long kx = lane < kCW ? sh.key[s][lane] : 0ull;
+      unsigned long long kbest;
+      wb = warp_first_max(kx, &kbest);
+    }
+    const int p_off = sh.idx[s][wb] - k;
+    double u[kNB];
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) u[d] = sh.piv[s][wb][d];
+    const unsigned um = sh.pivm[s][wb];
+    const bool zero = ((um >> k) & 1u) == 0u;
+    if (tid == 0) {
+      sh.pk[pp][k] = p_off;
+      sh.zp[pp][k] = zero ? 1 : 0;
+      if (zero && info == 0) info = j + 1;
+    }
+    double lsend = 0.0;
+    if (!zero) {
+      double rc = sh.prc[s][wb];
+      if (sh.pspec[s][wb]) rc = rcp_division(u[k]);  // uniform
+      if (i == k) {
+#pragma unroll
+        for (int d = 0; d < kNB; ++d)
+          if (d >= k) v[d] = u[d];
+      } else if (p_off != 0 && i == k + p_off) {
+#pragma unroll
+        for (int d = 0; d < kNB; ++d)
+          if (d >= k) v[d] = sh.row0[s][d];
+      }
+      if (i > k && i <= k + km) {
+        const double l = v[k] * rc;
+        v[k] = l;
+        lsend = l;
+#pragma unroll
+        for (int d = 0; d < kNB; ++d)
+          if (d > k) v[d] = upd(l, u[d], v[d], (um >> d) & 1u);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < kStreamers; ++r) {
+      if (!((rt.mask >> r) & 1u)) continue;  // uniform
+      st_async_b64(rt.rec[r] + (unsigned)(k * kCT + tid) * 8u, dbl_bits_w(lsend), rt.bar[r] + (unsigned)k * 8u);
+      if (tid == 0)
+        st_async_v2(rt.hdr[r] + (unsigned)k * 16u, (unsigned long long)(unsigned)p_off, zero ? 1ull : 0ull,
+                    rt.bar[r] + (unsigned)k * 8u);
+    }
+  }
+  if (mine) {
+#pragma unroll
+    for (int k = 0; k < kNB; ++k)
+      if (k < nc && i - k <= g.kl) blk[k * ldab + g.kv + i - k] = v[k];
+  }
+}
+
+// One step k of panel q applied to the thread's row of a block (registers w),
+// the pivot row and row j broadcast through bc (the step functions' order).
+template <int CW>
+__device__ __forceinline__ void apply_step_regs(const Geo &g, double (&w)[kNB], int i, int k, int km, int p, double l,
+                                                Bcast &bc, int bar, int &bpar) {
+  const int s = bpar;
+  bpar ^= 1;
+  if (i == k + p) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) bc.bu[s][d] = w[d];
+    bc.bum[s] = nz_mask(w);
+  }
+  if (i == k) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) bc.br0[s][d] = w[d];
+  }
+  bar_group<CW>(bar);
+  double u[kNB];
+#pragma unroll
+  for (int d = 0; d < kNB; ++d) u[d] = bc.bu[s][d];
+  const unsigned um = bc.bum[s];
+  if (i == k) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = u[d];
+  } else if (p != 0 && i == k + p) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = bc.br0[s][d];
+  }
+  if (i > k && i <= k + km) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = upd(l, u[d], w[d], (um >> d) & 1u);
+  }
+}
+
+// Blocks b >= kHandChain pass through an update CTA, which applies panels
+// p_first(b)..b-kHandChain.
+__device__ __forceinline__ bool handed_off_chain(const Geo &g, int b) {
+  return b >= kHandChain && p_first(g, b) <= b - kHandChain;
+}
+
+template <int CW>
+__global__ void __launch_bounds__(32 * (CW + 2), 1)
+    k_gbtrf_wide_chain(Geo g0, double *__restrict__ AB, int *__restrict__ ipiv, int *__restrict__ d_info,
+                       int *__restrict__ flags, const int *__restrict__ d_kl, const int *__restrict__ d_ku) {
+  constexpr int kCT = Lay<CW>::kCT, kCW = CW;
+  Geo g = g0;
+  if (d_kl != nullptr) {
+    // enqueued by the device-side dispatch: every CTA reads the decision and (kl, ku) alike
+    if (*(volatile const int *)(flags + 1) == 0) return;
+    g.kl = *d_kl;
+    g.ku = *d_ku;
+    g.kv = g.kl + g.ku;
+  }
+  extern __shared__ __align__(16) double smem[];
+  __shared__ StreamShared<CW> ss;
+  WideShared<CW, 1> &sh = ss.w;
+  int *err = flags;
+  int *panel_ready = flags + 2;
+  int *block_ready = flags + 2 + g.npan;
+  const long long bsz = (long long)kNB * g.ldab;
+  const unsigned blk_bytes = (unsigned)(bsz * sizeof(double));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // A: kPanelBufs block buffers; a streamer: kSlots block slots and its step records;
+  // update CTAs: kMaxActive block buffers
+  double *blocks = smem;
+  double *recs = smem + (size_t)kSlots * bsz;  // kRecDepth * kNB slots of kCT multipliers
+  auto buf = [&](int b) { return blocks + (long long)(b % kPanelBufs) * bsz; };
+  auto sbuf = [&](int b) { return blocks + (long long)((b - 1) % kSlots) * bsz; };
+  auto rslot = [](int q, int k) { return (q % kRecDepth) * kNB + k; };
+
+  if (tid == 0) {
+    for (int i = 0; i < kRing; ++i) {
+      mbar_init(&sh.mb_done[i], 1);
+      mbar_init(&ss.mb_blk[i], 1);
+      mbar_init(&ss.mb_afree[i], 1);
+      mbar_init(&ss.mb_pub[i], 1);
+    }
+    for (int i = 0; i < kRecDepth * kNB; ++i) mbar_init(&ss.mb_rec[i], 1);
+    for (int i = 0; i < kSlots; ++i) mbar_init(&ss.mb_in[i], 1);
+    sh.info = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  cluster_barrier();  // every CTA's barriers initialised before any remote operation
+
+  // a group's wait: every thread polls (a lone polling thread in an otherwise parked warp
+  // is slow to see the event), one barrier makes the outcome uniform
+  auto grp_wait = [&](auto ready, int bar_id) -> bool { return bar_and_group<CW>(bar_id, bounded_poll(ready, err)); };
+
+  if (blockIdx.x == 0) {
+    if (warp < kCW) {
+      // ---------------- A, group: panel p factored, its steps streamed to the streamers ----------------
+      int info = 0, bpar = 0;
+      load_block(g, AB, buf(0), 0, true, tid, kCT);
+      bar_compute<CW>();
+      for (int p = 0; p < g.npan; ++p) {
+        // block p+1 arrives from streamer 1 once panel p is applied to it
+        if (tid == 0 && p + 1 < g.npan)
+          mbar_expect_tx_local(&ss.mb_blk[p % kRing],
+                               (unsigned)(min(kNB, g.n - (p + 1) * kNB) * g.ldab * (long long)sizeof(double)));
+        RecTarget rt;
+        rt.mask = 0u;
+#pragma unroll
+        for (int r = 0; r < kStreamers; ++r) {
+          rt.rec[r] = cl_map(recs + (size_t)rslot(p, 0) * kCT, r + 1);
+          rt.hdr[r] = cl_map(&ss.rhdr[rslot(p, 0)][0], r + 1);
+          rt.bar[r] = cl_map(&ss.mb_rec[rslot(p, 0)], r + 1);
+          if (p + r + 1 < g.npan) rt.mask |= 1u << r;  // streamer r+1 applies panel p to block p+r+1
+        }
+        factor_panel_stream<CW>(g, buf(p), p, sh, bpar, info, rt);
+        if (tid == 0) {
+          sh.info = info;
+#pragma unroll
+          for (int k = 0; k < kNB; ++k) sh.pvr[p % kRing][k] = sh.pk[p & 1][k];
+        }
+        bar_compute<CW>();
+        if (tid == 0) mbar_arrive(&sh.mb_done[p % kRing]);  // the storer
+        if (p + 1 < g.npan) {
+          unsigned long long *mb = &ss.mb_blk[p % kRing];
+          const unsigned par = ring_parity(p, kRing);
+          if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarA)) break;
+        }
+      }
+    } else if (warp == kCW) {
+      // ---------------- A, publisher: a finished panel's diagonal, multipliers and pivots ----------------
+      for (int p = 0; p < g.npan; ++p) {
+        unsigned long long *mb = &sh.mb_done[p % kRing];
+        if (!io_wait_all([&] { return mbar_try_wait(mb, ring_parity(p, kRing)); }, err)) break;
+        const int c0 = p * kNB, nc = min(kNB, g.n - c0);
+        const double *src = buf(p);
+        double *dst = AB + (long long)c0 * g.ldab;
+        const int ld = (int)g.ldab;
+        for (int k = 0; k < nc; ++k)
+          for (int rr = g.kv + lane; rr <= g.kv + g.kl; rr += 32) dst[k * ld + rr] = src[k * ld + rr];
+        if (lane < nc) ipiv[c0 + lane] = c0 + lane + sh.pvr[p % kRing][lane] + 1;
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) {
+          st_release(panel_ready + p, 1);
+          mbar_arrive(&ss.mb_pub[p % kRing]);
+        }
+      }
+    } else if (warp == kCW + 1) {
+      // ---------------- A, storer: the whole finished block, then its buffer is free ----------------
+      for (int p = 0; p < g.npan; ++p) {
+        unsigned long long *mb = &ss.mb_pub[p % kRing];
+        if (!io_wait_all([&] { return mbar_try_wait(mb, ring_parity(p, kRing)); }, err)) break;
+        store_block(g, AB, buf(p), p, lane, 32);
+        __syncwarp();
+        // this buffer takes block p+3 next, which streamer 1 sends
+        if (p + 3 < g.npan && lane == 0) cl_arrive(&ss.mb_afree[p % kRing], 1);
+      }
+      // info is final once the last panel is done; the status reflects every CTA's waits
+      if (lane == 0) *d_info = ld_acquire(err) ? -BANDLU_ERR_TIMEOUT : sh.info;
+    }
+  } else if (blockIdx.x < kChainCTAs) {
+    const int r = blockIdx.x;  // streamer r: panel b-r to block b, then block b to CTA r-1
+    if (warp < kCW) {
+      int bpar = 0;
+      const int i = tid;
+      const int ld = (int)g.ldab;
+      for (int b = 1; b < g.npan; ++b) {
+        const int slot = (b - 1) % kSlots;
+        if (r < kStreamers && tid == 0) mbar_expect_tx_local(&ss.mb_in[slot], blk_bytes);
+        {
+          unsigned long long *mb = &ss.mb_in[slot];
+          const unsigned par = ring_parity(b - 1, kSlots);
+          if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) break;
+        }
+        const int q = b - r;
+        double *bx = sbuf(b);
+        const int c0b = b * kNB, ncb = min(kNB, g.n - c0b);
+        if (r == 1) {
+          // ---- streamer 1: panel b-1 streamed from A, the block written into A's buffer ----
+          // A's buffer of block b held block b-3: wait until its storer is done with it
+          if (b >= 3) {
+            unsigned long long *mb = &ss.mb_afree[(b - 3) % kRing];
+            const unsigned par = ring_parity(b - 3, kRing);
+            if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) break;
+          }
+          const unsigned dst = cl_map(buf(b), 0), dbar = cl_map(&ss.mb_blk[(b - 1) % kRing], 0);
+          // every value outside panel q's rows (band positions kv-4-d .. kv+kl-1-d of column d)
+          // is final already: it goes now, while the panel's steps arrive.  Each column's two
+          // runs go as bulk copies between 16-byte boundaries (thread 0), the at most two
+          // values cut off at each end of a run as 8-byte st.async (threads 1..); the band
+          // itself goes after the last step
+          if (tid < 1 + 4 * 2 * kNB) {
+            for (int d = 0; d < ncb; ++d) {
+              const int blo = g.kv - kNB - d, bhi = g.kv + g.kl - 1 - d;
+              const int runs[2][2] = {{0, blo}, {bhi + 1, ld}};  // [first, end) of each run
+#pragma unroll
+              for (int h = 0; h < 2; ++h) {
+                const int e0 = d * ld + runs[h][0], e1 = d * ld + runs[h][1];  // element range
+                if (e1 <= e0) continue;
+                const int a0 = (e0 + 1) & ~1, a1 = e1 & ~1;  // 16-byte aligned element range
+                if (a1 > a0) {
+                  if (tid == 0)
+                    asm volatile(
+                        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, "
+                        "[%3];" ::"r"(dst + (unsigned)a0 * 8u),
+                        "r"(smem_addr(bx + a0)), "r"((unsigned)(a1 - a0) * 8u), "r"(dbar)
+                        : "memory");
+                  const int t = 1 + (d * 2 + h) * 2;  // two threads per run for its cut-off ends
+                  if (tid == t && e0 < a0) st_async_b64(dst + (unsigned)e0 * 8u, dbl_bits_w(bx[e0]), dbar);
+                  if (tid == t + 1 && a1 < e1) st_async_b64(dst + (unsigned)a1 * 8u, dbl_bits_w(bx[a1]), dbar);
+                } else {
+                  const int t = 1 + (d * 2 + h) * 2;
+                  if (tid == t) st_async_b64(dst + (unsigned)e0 * 8u, dbl_bits_w(bx[e0]), dbar);
+                  if (tid == t + 1 && e0 + 1 < e1) st_async_b64(dst + (unsigned)(e0 + 1) * 8u, dbl_bits_w(bx[e0 + 1]), dbar);
+                }
+              }
+            }
+          }
+          const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
+          const int row = c0q + i;
+          const bool mine = i < g.kl + kNB && row < g.n;
+          double w[kNB];
+#pragma unroll
+          for (int d = 0; d < kNB; ++d) {
+            const int pos = g.kv + row - (c0b + d);
+            w[d] = (i < g.kl + kNB && d < ncb && pos >= 0) ? bx[d * ld + pos] : 0.0;
+          }
+          bool ok = true;
+#pragma unroll
+          for (int k = 0; k < kNB; ++k) {
+            if (k >= ncq) break;  // uniform
+            const int sl = rslot(q, k);
+            if (tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
+            unsigned long long *mb = &ss.mb_rec[sl];
+            const unsigned par = ring_parity(q, kRecDepth);
+            if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) {
+              ok = false;
+              break;
+            }
+            if (!ss.rhdr[sl][1]) {  // uniform: not a zero pivot
+              const double l = recs[(size_t)sl * kCT + i];
+              const int pk = (int)ss.rhdr[sl][0];
+              const int km = min(g.kl, g.n - 1 - (c0q + k));
+              double wm[kNB];
+#pragma unroll
+              for (int d = 0; d < kNB; ++d) wm[d] = w[d];
+              apply_step_regs<CW>(g, wm, i, k, km, pk, l, sh.bc[1], kBarB, bpar);
+              if (mine) {
+#pragma unroll
+                for (int d = 0; d < kNB; ++d) w[d] = wm[d];
+              }
+            }
+          }
+          if (!ok) break;
+          // panel q's rows of the block: one value per (row, column), from the row's thread
+          if (i < g.kl + kNB) {
+#pragma unroll
+            for (int d = 0; d < kNB; ++d) {
+              const int pos = g.kv - kNB + i - d;
+              if (d < ncb) st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(w[d]), dbar);
+            }
+          }
+        } else {
+          // ---- streamers 2..: panel b-r as it streams from A, the block to streamer r-1 ----
+          if (q >= 0) {
+            const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
+            const bool apply = q >= p_first(g, b);  // uniform
+            const int row = c0q + i;
+            const bool mine = i < g.kl + kNB && row < g.n;
+            double w[kNB];
+#pragma unroll
+            for (int d = 0; d < kNB; ++d) {
+              const int pos = g.kv + row - (c0b + d);
+              w[d] = (apply && mine && d < ncb && pos >= 0) ? bx[d * ld + pos] : 0.0;
+            }
+            bool ok = true;
+#pragma unroll
+            for (int k = 0; k < kNB; ++k) {
+              if (k >= ncq) break;  // uniform
+              const int sl = rslot(q, k);
+              if (tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
+              unsigned long long *mb = &ss.mb_rec[sl];
+              const unsigned par = ring_parity(q, kRecDepth);
+              if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) {
+                ok = false;
+                break;
+              }
+              if (apply && !ss.rhdr[sl][1]) {  // uniform
+                const double l = recs[(size_t)sl * kCT + i];
+                const int pk = (int)ss.rhdr[sl][0];
+                const int km = min(g.kl, g.n - 1 - (c0q + k));
+                apply_step_regs<CW>(g, w, i, k, km, pk, l, sh.bc[1], kBarB, bpar);
+              }
+            }
+            if (!ok) break;
+            if (apply && mine) {
+#pragma unroll
+              for (int d = 0; d < kNB; ++d) {
+                const int pos = g.kv + row - (c0b + d);
+                if (d < ncb && pos >= 0) bx[d * ld + pos] = w[d];
+              }
+            }
+          }
+          // into streamer r-1's slot, which held block b-kSlots: A must have factored it
+          if (b - kSlots >= 1) {
+            const int *f = panel_ready + (b - kSlots);
+            if (!grp_wait([&] { return ld_acquire(f) != 0; }, kBarB)) break;
+          }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the block's stores, before the copy
+          bar_group<CW>(kBarB);
+          if (tid == 0)
+            asm volatile(
+                "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    cl_map(sbuf(b), r - 1)),
+                "r"(smem_addr(bx)), "r"(blk_bytes), "r"(cl_map(&ss.mb_in[(b - 1) % kSlots], r - 1))
+                : "memory");
+        }
+      }
+    } else if (warp == kCW && r == kStreamers) {
+      // ---------------- last streamer, loader: blocks b >= 1 into its slots ----------------
+      for (int b = 1; b < g.npan; ++b) {
+        // the slot held block b-kSlots, passed on by now: A has factored it
+        if (b - kSlots >= 1) {
+          const int *f = panel_ready + (b - kSlots);
+          if (!io_wait_all([&] { return ld_acquire(f) != 0; }, err)) break;
+        }
+        double *dst = sbuf(b);
+        unsigned long long *ml = &ss.mb_in[(b - 1) % kSlots];
+        if (handed_off_chain(g, b)) {
+          const int *f = block_ready + b;
+          if (!io_wait_all([&] { return ld_acquire(f) != 0; }, err)) break;
+          if (g.vec && (b + 1) * kNB <= g.n) {
+            if (lane == 0) bulk_prefetch_block(g, AB, dst, b, ml);  // completes the phase itself
+            __syncwarp();
+            continue;
+          }
+          if (g.vec) {
+            io_prefetch_block(g, AB, dst, b);
+          } else {
+            load_block(g, AB, dst, b, false, lane, 32);
+          }
+        } else {
+          load_block(g, AB, dst, b, true, lane, 32);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(ml);
+      }
+    }
+  } else {
+    // ---------------- update CTAs: panels p_first(b)..b-kHandChain to their blocks ----------------
+    if (warp >= kCW) return;
+    const int G = gridDim.x - kChainCTAs, u = blockIdx.x - kChainCTAs;
+    int bpar = 0;
+    for (int p = 0; p + kHandChain < g.npan; ++p) {
+      const int lo = p + kHandChain, hi = b_last(g, p);
+      const int b0 = lo + ((u - (lo - kHandChain)) % G + G) % G;
+      if (b0 > hi) continue;
+      const int *f = panel_ready + p;
+      if (!compute_wait<CW, 1>([&] { return ld_acquire(f) != 0; }, err, sh)) break;
+      const int c0q = p * kNB, ncq = min(kNB, g.n - c0q);
+      if (tid < kNB) {
+        const int k = tid;
+        sh.pk[0][k] = k < ncq ? __ldcg(ipiv + c0q + k) - 1 - (c0q + k) : 0;
+        sh.zp[0][k] = k < ncq ? (nz(__ldcg(AB + (long long)(c0q + k) * g.ldab + g.kv)) ? 0 : 1) : 1;
+      }
+      double lr[1][kNB];
+#pragma unroll
+      for (int k = 0; k < kNB; ++k) {
+        const int t = tid - k;
+        lr[0][k] = (k < ncq && t >= 1 && t <= min(g.kl, g.n - 1 - (c0q + k)))
+                       ? __ldcg(AB + (long long)(c0q + k) * g.ldab + g.kv + t)
+                       : 0.0;
+      }
+      bar_compute<CW>();
+      for (int b = b0; b <= hi; b += G) {
+        double *blk = blocks + (long long)(((b - kHandChain) / G) % kMaxActive) * bsz;
+        if (p == p_first(g, b)) {
+          load_block(g, AB, blk, b, true, tid, kCT);
+          bar_compute<CW>();
+        }
+        apply_panel<CW, 1>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh.bc[0], tid, kBarA, bpar);
+        bar_compute<CW>();
+        if (p == b - kHandChain) {
+          store_block(g, AB, blk, b, tid, kCT);
+          __threadfence();
+          bar_compute<CW>();
+          if (tid == 0) st_release(block_ready + b, 1);
+        }
+      }
+    }
+    return;
+  }
+  // after a wait gave up, let a bulk copy or st.async still in flight land
+  if (ld_relaxed(err) != 0) {
+    const long long t0 = clock64();
+    while (clock64() - t0 < 4000000) {
+    }
+  }
+  // the cluster's CTAs leave together: no distributed-shared-memory access or bulk copy
+  // can reach a CTA that has exited
+  cluster_barrier();
+}
+// Shared memory of the chain kernel: A three blocks, a streamer kSlots blocks and its
+// step records, update CTAs two blocks.
+size_t stream_smem(long long ldab, int cw) {
+  const size_t bs = (size_t)kNB * (size_t)ldab;
+  const size_t need_a = (size_t)kPanelBufs * bs;
+  const size_t need_b = (size_t)kSlots * bs + (size_t)kRecDepth * kNB * 32 * (size_t)cw;
+  const size_t need_u = (size_t)kMaxActive * bs;
+  return std::max(need_a, std::max(need_b, need_u)) * sizeof(double);
+}
+
+// Cooperative launch with clusters of kChainCTAs.  prepare() answers with the grid: as
+// many whole clusters as can be resident at once (up to sms / kChainCTAs), 0 when fewer
+// than two fit, -1 on a CUDA error.  The answer is cached per (device, sms, shared
+// memory), so a call made during stream capture after a first call outside it issues no
+// query.
+template <int CW>
+struct StreamLaunch {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute at[2];
+  int prepare(int sms, size_t smem, cudaStream_t s) {
+    if (!allow_dynamic_smem(reinterpret_cast<const void *>(k_gbtrf_wide_chain<CW>), 200 * 1024)) return -1;
+    const int want = (sms / kChainCTAs) * kChainCTAs;
+    if (want < 2 * kChainCTAs) return 0;
+    cfg.gridDim = dim3((unsigned)want);
+    cfg.blockDim = dim3(32 * (CW + 2));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = kChainCTAs;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeCooperative;
+    at[1].val.cooperative = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+    static std::mutex mu;
+    static std::map<std::tuple<int, int, size_t>, int> grids;
+    const auto key = std::make_tuple(dev, want, smem);
+    int grid = 0;
+    {
+      std::lock_guard<std::mutex> lock(mu);
+      const auto it = grids.find(key);
+      if (it != grids.end()) grid = it->second;
+    }
+    if (grid == 0) {
+      int clusters = 0;
+      if (cudaOccupancyMaxActiveClusters(&clusters, k_gbtrf_wide_chain<CW>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        clusters = 0;
+      }
+      grid = std::min(clusters, want / kChainCTAs) * kChainCTAs;
+      if (grid < 2 * kChainCTAs) grid = -2;  // cached "does not fit"
+      std::lock_guard<std::mutex> lock(mu);
+      grids[key] = grid;
+    }
+    if (grid < 0) return 0;
+    cfg.gridDim = dim3((unsigned)grid);
+    return grid;
+  }
+  int launch(const Geo &g, double *AB, int *ipiv, int *d_info, int *flags, const int *d_kl, const int *d_ku) {
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    Geo gg = g;
+    if (cudaLaunchKernelEx(&cfg, k_gbtrf_wide_chain<CW>, gg, AB, ipiv, d_info, flags, d_kl, d_ku) != cudaSuccess)
+      return BANDLU_ERR_CUDA;
+    return BANDLU_OK;
+  }
+};
+
+// BANDLU_WIDE_PAIR=1 in the environment selects the cluster pair where the chain would
+// run (read once): the comparison the chain is measured against.
+bool chain_disabled() {
+  static const bool off = [] {
+    const char *v = std::getenv("BANDLU_WIDE_PAIR");
+    return v != nullptr && v[0] == '1';
+  }();
+  return off;
+}
