@@ -102,7 +102,8 @@ struct RecTarget {
 // factor_panel for one row per thread, streaming each step's multipliers to the streamers.
 template <int CW>
 __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared<CW, 1> &sh, int &bpar, int &info,
-                                    const RecTarget &rt) {
+                                    const RecTarget &rt, double *__restrict__ AB, int *__restrict__ ipiv,
+                                    double &lastl) {
   constexpr int kCT = Lay<CW>::kCT, kCW = CW;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int c0 = p * kNB, nc = min(kNB, g.n - c0);
@@ -110,6 +111,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
   const int pp = p & 1;
   const int i = tid, row = c0 + i;
   const bool mine = i < g.kl + kNB && row < g.n;
+  double *abp = AB + (long long)c0 * g.ldab;
   double v[kNB];
 #pragma unroll
   for (int k = 0; k < kNB; ++k) v[k] = (mine && k < nc && i - k <= g.kl) ? blk[k * ldab + g.kv + i - k] : 0.0;
@@ -157,6 +159,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
       if (zero && info == 0) info = j + 1;
     }
     double lsend = 0.0;
+    lastl = 0.0;
     if (!zero) {
       double rc = sh.prc[s][wb];
       if (sh.pspec[s][wb]) rc = rcp_division(u[k]);  // uniform
@@ -173,14 +176,20 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
         const double l = v[k] * rc;
         v[k] = l;
         lsend = l;
+        lastl = l;
 #pragma unroll
         for (int d = 0; d < kNB; ++d)
           if (d > k) v[d] = upd(l, u[d], v[d], (um >> d) & 1u);
       }
     }
+    // column k is final now (later interchanges touch columns k+1.. only): what the update
+    // CTAs read of it, the diagonal and the multipliers (band rows kv..kv+kl), goes straight
+    // into AB, so the publisher only has to release it once the group has arrived
+    if (mine && i >= k && i - k <= g.kl) abp[k * ldab + g.kv + i - k] = v[k];
 #pragma unroll
     for (int r = 0; r < kStreamers; ++r) {
       if (!((rt.mask >> r) & 1u)) continue;  // uniform
+      if (r == 0 && k == nc - 1) continue;    // A applies its panel's last step to block p+1 itself
       st_async_b64(rt.rec[r] + (unsigned)(k * kCT + tid) * 8u, dbl_bits_w(lsend), rt.bar[r] + (unsigned)k * 8u);
       if (tid == 0)
         st_async_v2(rt.hdr[r] + (unsigned)k * 16u, (unsigned long long)(unsigned)p_off, zero ? 1ull : 0ull,
@@ -191,6 +200,11 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
 #pragma unroll
     for (int k = 0; k < kNB; ++k)
       if (k < nc && i - k <= g.kl) blk[k * ldab + g.kv + i - k] = v[k];
+  }
+  if (tid == 0) {
+#pragma unroll
+    for (int k = 0; k < kNB; ++k)
+      if (k < nc) ipiv[c0 + k] = c0 + k + sh.pk[pp][k] + 1;
   }
 }
 
@@ -254,7 +268,6 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
   int *panel_ready = flags + 2;
   int *block_ready = flags + 2 + g.npan;
   const long long bsz = (long long)kNB * g.ldab;
-  const unsigned blk_bytes = (unsigned)(bsz * sizeof(double));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // A: kPanelBufs block buffers; a streamer: kSlots block slots and its step records;
   // update CTAs: kMaxActive block buffers
@@ -302,7 +315,8 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           rt.bar[r] = cl_map(&ss.mb_rec[rslot(p, 0)], r + 1);
           if (p + r + 1 < g.npan) rt.mask |= 1u << r;  // streamer r+1 applies panel p to block p+r+1
         }
-        factor_panel_stream<CW>(g, buf(p), p, sh, bpar, info, rt);
+        double lastl;
+        factor_panel_stream<CW>(g, buf(p), p, sh, bpar, info, rt, AB, ipiv, lastl);
         if (tid == 0) {
           sh.info = info;
 #pragma unroll
@@ -314,26 +328,45 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           unsigned long long *mb = &ss.mb_blk[p % kRing];
           const unsigned par = ring_parity(p, kRing);
           if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarA)) break;
+          // block p+1 holds panel p's steps but the last: that one is applied here, from the
+          // pivot and the multipliers this group has just formed
+          const int c0 = p * kNB, nc = min(kNB, g.n - c0), kk = nc - 1;
+          if (!sh.zp[p & 1][kk]) {  // uniform
+            const int i = tid, row = c0 + i;
+            const bool mine = i < g.kl + kNB && row < g.n;
+            const int c0b = (p + 1) * kNB, ncb = min(kNB, g.n - c0b);
+            double *bx = buf(p + 1);
+            double w[kNB];
+#pragma unroll
+            for (int d = 0; d < kNB; ++d) {
+              const int pos = g.kv + row - (c0b + d);
+              w[d] = (mine && d < ncb && pos >= 0) ? bx[d * (int)g.ldab + pos] : 0.0;
+            }
+            const int km = min(g.kl, g.n - 1 - (c0 + kk));
+            apply_step_regs<CW>(g, w, i, kk, km, sh.pk[p & 1][kk], lastl, sh.bc[0], kBarA, bpar);
+            if (mine) {
+#pragma unroll
+              for (int d = 0; d < kNB; ++d) {
+                const int pos = g.kv + row - (c0b + d);
+                if (d < ncb && pos >= 0) bx[d * (int)g.ldab + pos] = w[d];
+              }
+            }
+            bar_compute<CW>();
+          }
         }
       }
     } else if (warp == kCW) {
-      // ---------------- A, publisher: a finished panel's diagonal, multipliers and pivots ----------------
+      // ---------------- A, publisher: panel p's diagonal, multipliers and pivots released ----------------
+      // group A stored them to AB before its arrival on mb_done; that arrival (release), this
+      // warp's acquire and the release below carry them to every CTA that acquires panel_ready
       for (int p = 0; p < g.npan; ++p) {
         unsigned long long *mb = &sh.mb_done[p % kRing];
         if (!io_wait_all([&] { return mbar_try_wait(mb, ring_parity(p, kRing)); }, err)) break;
-        const int c0 = p * kNB, nc = min(kNB, g.n - c0);
-        const double *src = buf(p);
-        double *dst = AB + (long long)c0 * g.ldab;
-        const int ld = (int)g.ldab;
-        for (int k = 0; k < nc; ++k)
-          for (int rr = g.kv + lane; rr <= g.kv + g.kl; rr += 32) dst[k * ld + rr] = src[k * ld + rr];
-        if (lane < nc) ipiv[c0 + lane] = c0 + lane + sh.pvr[p % kRing][lane] + 1;
-        __threadfence();
-        __syncwarp();
         if (lane == 0) {
           st_release(panel_ready + p, 1);
           mbar_arrive(&ss.mb_pub[p % kRing]);
         }
+        __syncwarp();
       }
     } else if (warp == kCW + 1) {
       // ---------------- A, storer: the whole finished block, then its buffer is free ----------------
@@ -356,69 +389,106 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
       const int ld = (int)g.ldab;
       for (int b = 1; b < g.npan; ++b) {
         const int slot = (b - 1) % kSlots;
-        if (r < kStreamers && tid == 0) mbar_expect_tx_local(&ss.mb_in[slot], blk_bytes);
+        const int c0b = b * kNB, ncb = min(kNB, g.n - c0b);
+        const unsigned bytes = (unsigned)(ncb * ld * 8);  // what a block's move carries
+        if (r < kStreamers && tid == 0) mbar_expect_tx_local(&ss.mb_in[slot], bytes);
         {
           unsigned long long *mb = &ss.mb_in[slot];
           const unsigned par = ring_parity(b - 1, kSlots);
           if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) break;
         }
         const int q = b - r;
+        const bool apply = q >= 0 && q >= p_first(g, b);  // uniform
         double *bx = sbuf(b);
-        const int c0b = b * kNB, ncb = min(kNB, g.n - c0b);
+        // where the block goes: A's buffer (which held block b-3: its storer must be done), or
+        // streamer r-1's slot (which held block b-kSlots: A must have factored it)
+        unsigned dst, dbar;
         if (r == 1) {
-          // ---- streamer 1: panel b-1 streamed from A, the block written into A's buffer ----
-          // A's buffer of block b held block b-3: wait until its storer is done with it
           if (b >= 3) {
             unsigned long long *mb = &ss.mb_afree[(b - 3) % kRing];
             const unsigned par = ring_parity(b - 3, kRing);
             if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) break;
           }
-          const unsigned dst = cl_map(buf(b), 0), dbar = cl_map(&ss.mb_blk[(b - 1) % kRing], 0);
-          // every value outside panel q's rows (band positions kv-4-d .. kv+kl-1-d of column d)
-          // is final already: it goes now, while the panel's steps arrive.  Each column's two
-          // runs go as bulk copies between 16-byte boundaries (thread 0), the at most two
-          // values cut off at each end of a run as 8-byte st.async (threads 1..); the band
-          // itself goes after the last step
-          if (tid < 1 + 4 * 2 * kNB) {
-            for (int d = 0; d < ncb; ++d) {
-              const int blo = g.kv - kNB - d, bhi = g.kv + g.kl - 1 - d;
-              const int runs[2][2] = {{0, blo}, {bhi + 1, ld}};  // [first, end) of each run
-#pragma unroll
-              for (int h = 0; h < 2; ++h) {
-                const int e0 = d * ld + runs[h][0], e1 = d * ld + runs[h][1];  // element range
-                if (e1 <= e0) continue;
-                const int a0 = (e0 + 1) & ~1, a1 = e1 & ~1;  // 16-byte aligned element range
-                if (a1 > a0) {
-                  if (tid == 0)
-                    asm volatile(
-                        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, "
-                        "[%3];" ::"r"(dst + (unsigned)a0 * 8u),
-                        "r"(smem_addr(bx + a0)), "r"((unsigned)(a1 - a0) * 8u), "r"(dbar)
-                        : "memory");
-                  const int t = 1 + (d * 2 + h) * 2;  // two threads per run for its cut-off ends
-                  if (tid == t && e0 < a0) st_async_b64(dst + (unsigned)e0 * 8u, dbl_bits_w(bx[e0]), dbar);
-                  if (tid == t + 1 && a1 < e1) st_async_b64(dst + (unsigned)a1 * 8u, dbl_bits_w(bx[a1]), dbar);
-                } else {
-                  const int t = 1 + (d * 2 + h) * 2;
-                  if (tid == t) st_async_b64(dst + (unsigned)e0 * 8u, dbl_bits_w(bx[e0]), dbar);
-                  if (tid == t + 1 && e0 + 1 < e1) st_async_b64(dst + (unsigned)(e0 + 1) * 8u, dbl_bits_w(bx[e0 + 1]), dbar);
-                }
-              }
+          dst = cl_map(buf(b), 0);
+          dbar = cl_map(&ss.mb_blk[(b - 1) % kRing], 0);
+        } else {
+          if (b - kSlots >= 1) {
+            const int *f = panel_ready + (b - kSlots);
+            if (!grp_wait([&] { return ld_acquire(f) != 0; }, kBarB)) break;
+          }
+          dst = cl_map(sbuf(b), r - 1);
+          dbar = cl_map(&ss.mb_in[(b - 1) % kSlots], r - 1);
+        }
+        // panel q's rows of the block (band positions kv-4r-d .. kv-4r+kl+3-d of column d) change
+        // here; every other value is final for this move and goes now.  Between the bands the
+        // block is ncb+1 runs (a column's tail and the next column's head are contiguous); run
+        // j goes from warp j: a bulk copy between 16-byte boundaries (lane 0), the at most one
+        // value cut off at each end as an 8-byte st.async (lanes 1 and 2)
+        const int boff = g.kv - kNB * r;  // band position of row 4q, column 0
+        auto band = [&](int d, int &lo, int &hi) {  // band of column d, [lo, hi]; lo > hi: none
+          lo = ld;
+          hi = ld - 1;
+          if (apply) {
+            const int l0 = max(0, boff - d), h0 = min(ld - 1, boff + g.kl + kNB - 1 - d);
+            if (h0 >= l0) {
+              lo = l0;
+              hi = h0;
             }
           }
+        };
+        for (int j = warp; j <= ncb; j += kCW) {
+          int e0, e1;  // element range of run j
+          if (j == 0) {
+            int lo, hi;
+            band(0, lo, hi);
+            e0 = 0;
+            e1 = lo;
+          } else {
+            int lo, hi;
+            band(j - 1, lo, hi);
+            e0 = (j - 1) * ld + hi + 1;
+            if (j < ncb) {
+              int lo2, hi2;
+              band(j, lo2, hi2);
+              e1 = j * ld + lo2;
+            } else {
+              e1 = ncb * ld;
+            }
+          }
+          if (e1 > e0) {
+            const int a0 = (e0 + 1) & ~1, a1 = e1 & ~1;  // 16-byte aligned element range
+            if (a1 > a0) {
+              if (lane == 0)
+                asm volatile(
+                    "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                        dst + (unsigned)a0 * 8u),
+                    "r"(smem_addr(bx + a0)), "r"((unsigned)(a1 - a0) * 8u), "r"(dbar)
+                    : "memory");
+              if (lane == 1 && e0 < a0) st_async_b64(dst + (unsigned)e0 * 8u, dbl_bits_w(bx[e0]), dbar);
+              if (lane == 2 && a1 < e1) st_async_b64(dst + (unsigned)a1 * 8u, dbl_bits_w(bx[a1]), dbar);
+            } else {
+              if (lane == 1) st_async_b64(dst + (unsigned)e0 * 8u, dbl_bits_w(bx[e0]), dbar);
+              if (lane == 2 && e0 + 1 < e1) st_async_b64(dst + (unsigned)(e0 + 1) * 8u, dbl_bits_w(bx[e0 + 1]), dbar);
+            }
+          }
+        }
+        if (q >= 0) {
+          // panel q as its steps stream from A (streamer 1 leaves the last one to A); the
+          // records are taken whether or not the panel reaches this block
           const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
+          const int nsteps = r == 1 ? ncq - 1 : ncq;
           const int row = c0q + i;
           const bool mine = i < g.kl + kNB && row < g.n;
           double w[kNB];
 #pragma unroll
           for (int d = 0; d < kNB; ++d) {
-            const int pos = g.kv + row - (c0b + d);
-            w[d] = (i < g.kl + kNB && d < ncb && pos >= 0) ? bx[d * ld + pos] : 0.0;
+            const int pos = boff + i - d;
+            w[d] = (apply && i < g.kl + kNB && d < ncb && pos >= 0 && pos < ld) ? bx[d * ld + pos] : 0.0;
           }
           bool ok = true;
 #pragma unroll
           for (int k = 0; k < kNB; ++k) {
-            if (k >= ncq) break;  // uniform
+            if (k >= nsteps) break;  // uniform
             const int sl = rslot(q, k);
             if (tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
             unsigned long long *mb = &ss.mb_rec[sl];
@@ -427,7 +497,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
               ok = false;
               break;
             }
-            if (!ss.rhdr[sl][1]) {  // uniform: not a zero pivot
+            if (apply && !ss.rhdr[sl][1]) {  // uniform
               const double l = recs[(size_t)sl * kCT + i];
               const int pk = (int)ss.rhdr[sl][0];
               const int km = min(g.kl, g.n - 1 - (c0q + k));
@@ -442,68 +512,14 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
             }
           }
           if (!ok) break;
-          // panel q's rows of the block: one value per (row, column), from the row's thread
-          if (i < g.kl + kNB) {
+          // the band: one value per (row, column), from the row's thread
+          if (apply && i < g.kl + kNB) {
 #pragma unroll
             for (int d = 0; d < kNB; ++d) {
-              const int pos = g.kv - kNB + i - d;
-              if (d < ncb) st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(w[d]), dbar);
+              const int pos = boff + i - d;
+              if (d < ncb && pos >= 0 && pos < ld) st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(w[d]), dbar);
             }
           }
-        } else {
-          // ---- streamers 2..: panel b-r as it streams from A, the block to streamer r-1 ----
-          if (q >= 0) {
-            const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
-            const bool apply = q >= p_first(g, b);  // uniform
-            const int row = c0q + i;
-            const bool mine = i < g.kl + kNB && row < g.n;
-            double w[kNB];
-#pragma unroll
-            for (int d = 0; d < kNB; ++d) {
-              const int pos = g.kv + row - (c0b + d);
-              w[d] = (apply && mine && d < ncb && pos >= 0) ? bx[d * ld + pos] : 0.0;
-            }
-            bool ok = true;
-#pragma unroll
-            for (int k = 0; k < kNB; ++k) {
-              if (k >= ncq) break;  // uniform
-              const int sl = rslot(q, k);
-              if (tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
-              unsigned long long *mb = &ss.mb_rec[sl];
-              const unsigned par = ring_parity(q, kRecDepth);
-              if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) {
-                ok = false;
-                break;
-              }
-              if (apply && !ss.rhdr[sl][1]) {  // uniform
-                const double l = recs[(size_t)sl * kCT + i];
-                const int pk = (int)ss.rhdr[sl][0];
-                const int km = min(g.kl, g.n - 1 - (c0q + k));
-                apply_step_regs<CW>(g, w, i, k, km, pk, l, sh.bc[1], kBarB, bpar);
-              }
-            }
-            if (!ok) break;
-            if (apply && mine) {
-#pragma unroll
-              for (int d = 0; d < kNB; ++d) {
-                const int pos = g.kv + row - (c0b + d);
-                if (d < ncb && pos >= 0) bx[d * ld + pos] = w[d];
-              }
-            }
-          }
-          // into streamer r-1's slot, which held block b-kSlots: A must have factored it
-          if (b - kSlots >= 1) {
-            const int *f = panel_ready + (b - kSlots);
-            if (!grp_wait([&] { return ld_acquire(f) != 0; }, kBarB)) break;
-          }
-          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the block's stores, before the copy
-          bar_group<CW>(kBarB);
-          if (tid == 0)
-            asm volatile(
-                "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                    cl_map(sbuf(b), r - 1)),
-                "r"(smem_addr(bx)), "r"(blk_bytes), "r"(cl_map(&ss.mb_in[(b - 1) % kSlots], r - 1))
-                : "memory");
         }
       }
     } else if (warp == kCW && r == kStreamers) {
@@ -546,7 +562,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
       const int b0 = lo + ((u - (lo - kHandChain)) % G + G) % G;
       if (b0 > hi) continue;
       const int *f = panel_ready + p;
-      if (!compute_wait<CW, 1>([&] { return ld_acquire(f) != 0; }, err, sh)) break;
+      if (!bar_and_group<CW>(kBarA, bounded_poll([&] { return ld_acquire(f) != 0; }, err))) break;
       const int c0q = p * kNB, ncq = min(kNB, g.n - c0q);
       if (tid < kNB) {
         const int k = tid;
