@@ -8,10 +8,23 @@
 //
 //  * CTA 0 (A) only factors: block p arrives with panels 0..p-1 applied, group A
 //    factors it, and after every column step each thread sends its row's
-//    multiplier (thread 0 also the step's pivot offset and zero flag) into the
-//    streamers' shared memory with one 8-byte st.async per streamer, completing
-//    a transaction count on that streamer's barrier of the step.  A storer warp
-//    writes finished panels to AB and publishes them.
+//    multiplier (thread 0 also the step's pivot offset and zero flag) into
+//    streamer 1's shared memory with one 8-byte st.async, completing a
+//    transaction count on streamer 1's barrier of the step.  A forwarder warp on
+//    streamer r (r < kStreamers) passes each step's records on to streamer r+1
+//    with one bulk copy once they have arrived: only streamer 1 is on A's path
+//    (its block comes back next), the others have a panel or more in hand.  A
+//    storer warp writes finished panels to AB and publishes them.
+//  * In a column step only the next column's update is on the path to the
+//    next pivot search; the step's update of the columns after it is issued in
+//    the next step, beside its reciprocal and argmax (integer and FP32 work),
+//    before anything reads those columns.
+//  * Streamer 1 applies the first kNB-1 steps of panel p to block p+1; the
+//    last one is applied by A as it starts panel p+1, straight from the block
+//    that arrived: each thread reads the step's pivot row and row j from shared
+//    memory and takes its own row's multiplier from the thread that held that
+//    row in panel p (four rows lower), updates column 0 at once and the other
+//    columns through the deferred update of step 0.
 //  * CTA r (streamer r, 1 <= r <= kStreamers) receives every block b from CTA
 //    r+1 (streamer kStreamers from its loader, which takes the block from AB once
 //    an update CTA has applied panels p_first(b)..b-kHandChain), applies panel
@@ -47,6 +60,7 @@ struct StreamShared {
   unsigned long long mb_afree[kRing];          // streamer 1: A's buffer of block p stored (A's storer), event p
   unsigned long long mb_pub[kRing];            // A: panel p published (publisher), event p
   alignas(16) unsigned long long rhdr[kRecDepth * kNB][2];  // streamer: pivot offset and zero flag of (q, k)
+  double lm[32 * CW];  // A: each thread's multiplier of the last step of the panel just factored
 };
 
 __device__ __forceinline__ unsigned long long dbl_bits_w(double x) {
@@ -90,20 +104,23 @@ __device__ __forceinline__ bool io_wait_all(F ready, int *err) {
   return __all_sync(FULL, ok);
 }
 
-// Where the records of panel p go on each streamer (cluster addresses); bit r-1
-// of mask: streamer r consumes panel p (block p+r exists).
+// Where the records of panel p go on streamer 1 (cluster addresses); send: block
+// p+1 exists, so streamer 1 (and its forwarder) takes panel p.
 struct RecTarget {
-  unsigned rec[kStreamers];  // multiplier slots of step 0 (step k: + k * kCT * 8)
-  unsigned hdr[kStreamers];  // header of step 0 (step k: + k * 16)
-  unsigned bar[kStreamers];  // barrier of step 0 (step k: + k * 8)
-  unsigned mask;
+  unsigned rec;  // multiplier slots of step 0 (step k: + k * kCT * 8)
+  unsigned hdr;  // header of step 0 (step k: + k * 16)
+  unsigned bar;  // barrier of step 0 (step k: + k * 8)
+  bool send;
 };
 
 // factor_panel for one row per thread, streaming each step's multipliers to the streamers.
+// fuse: block p holds panels 0..p-1 but for the last step of panel p-1, which is
+// applied here (multipliers in lm, pivot offset and zero flag in sh.pk / sh.zp of
+// panel p-1).  On return lm holds this panel's last-step multipliers.
 template <int CW>
 __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared<CW, 1> &sh, int &bpar, int &info,
                                     const RecTarget &rt, double *__restrict__ AB, int *__restrict__ ipiv,
-                                    double &lastl) {
+                                    double *lm, bool fuse) {
   constexpr int kCT = Lay<CW>::kCT, kCW = CW;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int c0 = p * kNB, nc = min(kNB, g.n - c0);
@@ -115,6 +132,45 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
   double v[kNB];
 #pragma unroll
   for (int k = 0; k < kNB; ++k) v[k] = (mine && k < nc && i - k <= g.kl) ? blk[k * ldab + g.kv + i - k] : 0.0;
+  // the previous step's multiplier, pivot row and its nonzero mask, for its deferred update
+  // of the columns after the next one (pact: this row took that update)
+  double pl = 0.0, pu[kNB];
+  unsigned pum = 0u;
+  bool pact = false;
+#pragma unroll
+  for (int d = 0; d < kNB; ++d) pu[d] = 0.0;
+  // panel p-1's last step (row jq = c0-1, pivot row jq+pq): interchange, then the update of
+  // rows jq+1..jq+kmq, i.e. threads 0..kmq-1 (held by threads 4..kmq+3 in panel p-1)
+  bool wrow = false;  // row jq of this block takes the pivot row (written after step 0's barrier)
+  double uq[kNB];
+#pragma unroll
+  for (int d = 0; d < kNB; ++d) uq[d] = 0.0;
+  if (fuse && !sh.zp[(p - 1) & 1][kNB - 1]) {  // uniform
+    const int pq = sh.pk[(p - 1) & 1][kNB - 1];
+    const int kmq = min(g.kl, g.n - c0);
+    double r0[kNB];
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) {
+      uq[d] = d < nc ? blk[d * ldab + g.kv + pq - 1 - d] : 0.0;
+      r0[d] = d < nc ? blk[d * ldab + g.kv - 1 - d] : 0.0;
+    }
+    if (pq != 0 && i == pq - 1) {
+#pragma unroll
+      for (int d = 0; d < kNB; ++d) v[d] = r0[d];
+    }
+    wrow = pq != 0;
+    if (i < kmq) {
+      const double l = lm[i + kNB];
+      const unsigned um = nz_mask(uq);
+      v[0] = upd(l, uq[0], v[0], um & 1u);
+      pl = l;
+      pact = true;
+#pragma unroll
+      for (int d = 0; d < kNB; ++d) pu[d] = uq[d];
+      pum = um;
+    }
+  }
+  double lastl = 0.0;
 #pragma unroll
   for (int k = 0; k < kNB; ++k) {
     if (k >= nc) break;
@@ -125,6 +181,14 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
     bool myspec;
     const double myr = rcp_rn_fast(v[k], &myspec);
     const unsigned long long key = (t >= 0 && t <= km) ? pivot_key(v[k], t == 0) : 0ull;
+    // step k-1's update of columns k+1.. (its update of column k is done): before this
+    // step publishes or interchanges anything, so every element still receives the
+    // steps in order
+    if (pact) {
+#pragma unroll
+      for (int d = 0; d < kNB; ++d)
+        if (d > k) v[d] = upd(pl, pu[d], v[d], (pum >> d) & 1u);
+    }
     unsigned long long kmax;
     const int wl = warp_first_max(key, &kmax);
     if (lane == wl) {
@@ -141,6 +205,11 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
       for (int d = 0; d < kNB; ++d) sh.row0[s][d] = v[d];
     }
     bar_compute<CW>();
+    if (k == 0 && wrow && tid == 0) {  // every thread has read row jq above
+#pragma unroll
+      for (int d = 0; d < kNB; ++d)
+        if (d < nc) blk[d * ldab + g.kv - 1 - d] = uq[d];
+    }
     int wb = 0;
     if constexpr (kCW <= 32) {
       const unsigned long long kx = lane < kCW ? sh.key[s][lane] : 0ull;
@@ -160,6 +229,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
     }
     double lsend = 0.0;
     lastl = 0.0;
+    pact = false;
     if (!zero) {
       double rc = sh.prc[s][wb];
       if (sh.pspec[s][wb]) rc = rcp_division(u[k]);  // uniform
@@ -177,23 +247,23 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
         v[k] = l;
         lsend = l;
         lastl = l;
+        if (k + 1 < kNB) v[k + 1] = upd(l, u[k + 1], v[k + 1], (um >> (k + 1)) & 1u);
+        pl = l;
+        pact = true;
 #pragma unroll
-        for (int d = 0; d < kNB; ++d)
-          if (d > k) v[d] = upd(l, u[d], v[d], (um >> d) & 1u);
+        for (int d = 0; d < kNB; ++d) pu[d] = u[d];
+        pum = um;
       }
     }
     // column k is final now (later interchanges touch columns k+1.. only): what the update
     // CTAs read of it, the diagonal and the multipliers (band rows kv..kv+kl), goes straight
     // into AB, so the publisher only has to release it once the group has arrived
     if (mine && i >= k && i - k <= g.kl) abp[k * ldab + g.kv + i - k] = v[k];
-#pragma unroll
-    for (int r = 0; r < kStreamers; ++r) {
-      if (!((rt.mask >> r) & 1u)) continue;  // uniform
-      if (r == 0 && k == nc - 1) continue;    // A applies its panel's last step to block p+1 itself
-      st_async_b64(rt.rec[r] + (unsigned)(k * kCT + tid) * 8u, dbl_bits_w(lsend), rt.bar[r] + (unsigned)k * 8u);
+    if (rt.send) {  // uniform; streamer 1 passes every step on, and applies all but the last
+      st_async_b64(rt.rec + (unsigned)(k * kCT + tid) * 8u, dbl_bits_w(lsend), rt.bar + (unsigned)k * 8u);
       if (tid == 0)
-        st_async_v2(rt.hdr[r] + (unsigned)k * 16u, (unsigned long long)(unsigned)p_off, zero ? 1ull : 0ull,
-                    rt.bar[r] + (unsigned)k * 8u);
+        st_async_v2(rt.hdr + (unsigned)k * 16u, (unsigned long long)(unsigned)p_off, zero ? 1ull : 0ull,
+                    rt.bar + (unsigned)k * 8u);
     }
   }
   if (mine) {
@@ -201,6 +271,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
     for (int k = 0; k < kNB; ++k)
       if (k < nc && i - k <= g.kl) blk[k * ldab + g.kv + i - k] = v[k];
   }
+  lm[tid] = lastl;  // read by panel p+1 after the group's next barrier
   if (tid == 0) {
 #pragma unroll
     for (int k = 0; k < kNB; ++k)
@@ -307,16 +378,11 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           mbar_expect_tx_local(&ss.mb_blk[p % kRing],
                                (unsigned)(min(kNB, g.n - (p + 1) * kNB) * g.ldab * (long long)sizeof(double)));
         RecTarget rt;
-        rt.mask = 0u;
-#pragma unroll
-        for (int r = 0; r < kStreamers; ++r) {
-          rt.rec[r] = cl_map(recs + (size_t)rslot(p, 0) * kCT, r + 1);
-          rt.hdr[r] = cl_map(&ss.rhdr[rslot(p, 0)][0], r + 1);
-          rt.bar[r] = cl_map(&ss.mb_rec[rslot(p, 0)], r + 1);
-          if (p + r + 1 < g.npan) rt.mask |= 1u << r;  // streamer r+1 applies panel p to block p+r+1
-        }
-        double lastl;
-        factor_panel_stream<CW>(g, buf(p), p, sh, bpar, info, rt, AB, ipiv, lastl);
+        rt.rec = cl_map(recs + (size_t)rslot(p, 0) * kCT, 1);
+        rt.hdr = cl_map(&ss.rhdr[rslot(p, 0)][0], 1);
+        rt.bar = cl_map(&ss.mb_rec[rslot(p, 0)], 1);
+        rt.send = p + 1 < g.npan;  // streamer 1 applies panel p to block p+1
+        factor_panel_stream<CW>(g, buf(p), p, sh, bpar, info, rt, AB, ipiv, ss.lm, p > 0);
         if (tid == 0) {
           sh.info = info;
 #pragma unroll
@@ -328,31 +394,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           unsigned long long *mb = &ss.mb_blk[p % kRing];
           const unsigned par = ring_parity(p, kRing);
           if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarA)) break;
-          // block p+1 holds panel p's steps but the last: that one is applied here, from the
-          // pivot and the multipliers this group has just formed
-          const int c0 = p * kNB, nc = min(kNB, g.n - c0), kk = nc - 1;
-          if (!sh.zp[p & 1][kk]) {  // uniform
-            const int i = tid, row = c0 + i;
-            const bool mine = i < g.kl + kNB && row < g.n;
-            const int c0b = (p + 1) * kNB, ncb = min(kNB, g.n - c0b);
-            double *bx = buf(p + 1);
-            double w[kNB];
-#pragma unroll
-            for (int d = 0; d < kNB; ++d) {
-              const int pos = g.kv + row - (c0b + d);
-              w[d] = (mine && d < ncb && pos >= 0) ? bx[d * (int)g.ldab + pos] : 0.0;
-            }
-            const int km = min(g.kl, g.n - 1 - (c0 + kk));
-            apply_step_regs<CW>(g, w, i, kk, km, sh.pk[p & 1][kk], lastl, sh.bc[0], kBarA, bpar);
-            if (mine) {
-#pragma unroll
-              for (int d = 0; d < kNB; ++d) {
-                const int pos = g.kv + row - (c0b + d);
-                if (d < ncb && pos >= 0) bx[d * (int)g.ldab + pos] = w[d];
-              }
-            }
-            bar_compute<CW>();
-          }
+          // block p+1 holds panel p's steps but the last, which the next factor_panel_stream applies
         }
       }
     } else if (warp == kCW) {
@@ -520,6 +562,44 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
               if (d < ncb && pos >= 0 && pos < ld) st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(w[d]), dbar);
             }
           }
+        }
+      }
+    } else if (warp == kCW + 1 && r < kStreamers) {
+      // ---------------- forwarder: panel q's step records on to streamer r+1 ----------------
+      // This streamer takes panel q iff block q+r exists, streamer r+1 iff block q+r+1 does.
+      // The group's thread 0 opens each step's phase (expect_tx) before its wait, except for
+      // the step streamer 1 leaves to A: that one is opened here.  Slot (q, k) held (q-5, k),
+      // whose phase this warp has seen complete; streamer r+1 has read its own copy of
+      // (q-5, k) before A can send (q, k), so both slots are free.
+      const unsigned rbytes = (unsigned)(kCT * 8);
+      bool ok = true;
+      for (int q = 0; ok && q + r < g.npan; ++q) {
+        const int ncq = min(kNB, g.n - q * kNB);
+        const bool fwd = q + r + 1 < g.npan;
+        for (int k = 0; k < ncq; ++k) {
+          const int sl = rslot(q, k);
+          unsigned long long *mb = &ss.mb_rec[sl];
+          if (r == 1 && k == ncq - 1 && lane == 0) mbar_expect_tx_local(mb, rbytes + 16u);
+          const unsigned par = ring_parity(q, kRecDepth);
+          if (!io_wait_all([&] { return cl_try_wait(mb, par); }, err)) {
+            ok = false;
+            break;
+          }
+          if (fwd && lane == 0) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            const unsigned rb = cl_map(mb, r + 1);
+            asm volatile(
+                "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    cl_map(recs + (size_t)sl * kCT, r + 1)),
+                "r"(smem_addr(recs + (size_t)sl * kCT)), "r"(rbytes), "r"(rb)
+                : "memory");
+            asm volatile(
+                "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    cl_map(&ss.rhdr[sl][0], r + 1)),
+                "r"(smem_addr(&ss.rhdr[sl][0])), "r"(16u), "r"(rb)
+                : "memory");
+          }
+          __syncwarp();
         }
       }
     } else if (warp == kCW && r == kStreamers) {
