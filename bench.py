@@ -60,6 +60,7 @@ KERNEL_SOURCES = {
     "k_gbtrf_window": ["gbtrf.cu", "common.cuh", "rcp.cuh", "sync.cuh", "regwin.cuh"],
     "k_gbtrf_regwin": ["gbtrf.cu", "common.cuh", "rcp.cuh", "sync.cuh", "regwin.cuh"],
     "k_detect_vec": ["detect.cu", "common.cuh"],
+    "k_detect_flat": ["detect.cu", "common.cuh"],
     "k_dense_to_band_tiled": ["convert.cu", "common.cuh"],
     "k_batch_scan_convert": ["batched.cu", "common.cuh", "regwin.cuh", "rcp.cuh"],
 }
@@ -743,7 +744,7 @@ def run_ours(args):
     elif dominant == "detect":
         roofline = {"bound": "hbm", "achieved": detect_bytes / t_detect / 1e9, "peak": hbm_peak, "unit": "GB/s",
                     "frac": detect_bytes / t_detect / 1e9 / hbm_peak,
-                    "traffic": profiled_traffic("k_detect_vec"), "kernel": "k_detect_vec", "peak_source": hbm_src}
+                    "traffic": profiled_traffic("k_detect_flat"), "kernel": "k_detect_flat", "peak_source": hbm_src}
     else:
         roofline = {"bound": "hbm", "achieved": convert_bytes / t_convert / 1e9, "peak": hbm_peak, "unit": "GB/s",
                     "frac": convert_bytes / t_convert / 1e9 / hbm_peak,
@@ -826,8 +827,8 @@ def run_ours(args):
             "cpu_baseline": cpu_baseline,
             "e2e": {"value": e2e_value, "unit": "GFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "ms_per_step": e2e_ms},
-            "gpu_launches": 3 * args.steps,
-            "gpu_launches_note": "per step: k_detect_vec, k_dense_to_band_tiled and the factorisation kernel",
+            "gpu_launches": 4 * args.steps,
+            "gpu_launches_note": "per step: k_detect_reset, k_detect_flat, k_dense_to_band_tiled and the factorisation kernel",
             "clocks": clocks,
             "wall_s_timed": t_wall1 - t_wall0,
             "workloads": others,

@@ -48,6 +48,25 @@ def test_detect_special_cases():
         assert detect_gpu(s.to(DEV)) == (n - 7, 0)
 
 
+@pytest.mark.parametrize("n", [1025, 2049])
+def test_detect_contiguous_odd_rows_ignore_padding(n):
+    """Rows of odd length n stored with lda = n+1 form one contiguous run of 16-byte vectors:
+    the padding column (garbage here, NaN and ones) is never counted, and a stray entry in the
+    matrix's very last element or first column of the last row is found."""
+    lda = n + 1
+    A = banded(n, 3, 5, seed=n, lda=lda)
+    A[:, n] = float("nan")
+    A[::2, n] = 1.0
+    assert detect_gpu(A.to(DEV), n, lda) == (3, 5)
+    B = A.clone()
+    B[n - 1, n - 1] = 0.0
+    B[0, n - 1] = 2.0                      # ku = n-1
+    assert detect_gpu(B.to(DEV), n, lda) == (3, n - 1)
+    C = A.clone()
+    C[n - 1, 0] = -1.0                     # kl = n-1
+    assert detect_gpu(C.to(DEV), n, lda) == (n - 1, 5)
+
+
 @pytest.mark.parametrize("n,lda", [(100, 101), (99, 100), (99, 99), (1000, 1003), (2048, 2050)])
 def test_detect_lda_padding_and_scalar_path(n, lda):
     A = banded(n, 4, 9, seed=n, lda=lda)
