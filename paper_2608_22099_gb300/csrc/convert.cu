@@ -6,22 +6,28 @@
 // exactly like that run, gathers the band part of rows j0-ku .. j0+T-1+kl of A
 // into it (each row's band segment is contiguous in A, so a warp reads it with
 // consecutive addresses), and streams the tile out with consecutive stores.
-// Only band entries of A are read; every AB entry is written.
+// Only band entries of A are read; every AB entry is written.  The gather is
+// issued as 8-byte cp.async copies, so a warp has all its rows in flight at once
+// instead of one load-store round trip per row; the zero fill touches only the
+// tile positions the gather does not write (fill rows, band rows outside the
+// matrix), so the two never meet.
 #include "common.cuh"
 
 namespace bandlu {
 namespace {
 
-__global__ void __launch_bounds__(256) k_dense_to_band_tiled(const double *__restrict__ A, long long lda, long long n,
-                                                             int kl, int ku, double *__restrict__ AB, long long ldab,
-                                                             int T) {
-  extern __shared__ double tile[];  // T * ldab, tile[c*ldab + r] = AB(r, j0+c)
-  const long long kv = (long long)kl + ku;
-  const long long j0 = (long long)blockIdx.x * T;
-  const int tcols = (int)min((long long)T, n - j0);
-  const long long tsize = (long long)tcols * ldab;
-  for (long long e = threadIdx.x; e < tsize; e += blockDim.x) tile[e] = 0.0;
-  __syncthreads();
+// Fills the shared tile of output columns [j0, j0+tcols) (tile[c*ldab + r] = AB(r, j0+c))
+// and returns after the block's barrier that makes it complete.
+__device__ __forceinline__ void fill_band_tile(const double *__restrict__ A, long long lda, long long n, long long kl,
+                                               long long ku, long long j0, int tcols, long long ldab, double *tile) {
+  const long long kv = kl + ku;
+  const int L = (int)ldab;
+  const int tsize = tcols * L;
+  for (int e = threadIdx.x; e < tsize; e += blockDim.x) {
+    const int c = e / L, r = e - c * L;
+    const long long i = j0 + c - kv + r;
+    if (r < kl || r > kv + kl || i < 0 || i >= n) tile[e] = 0.0;
+  }
   const long long i_lo = max(0ll, j0 - ku);
   const long long i_hi = min(n - 1, j0 + tcols - 1 + kl);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
@@ -29,10 +35,22 @@ __global__ void __launch_bounds__(256) k_dense_to_band_tiled(const double *__res
     const long long c_lo = max(j0, i - kl);
     const long long c_hi = min(min(j0 + tcols - 1, i + ku), n - 1);
     for (long long c = c_lo + lane; c <= c_hi; c += 32) {
-      tile[(c - j0) * ldab + (kv + i - c)] = A[i * lda + c];
+      const unsigned dst = (unsigned)__cvta_generic_to_shared(tile + (c - j0) * ldab + (kv + i - c));
+      asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(dst), "l"(A + i * lda + c) : "memory");
     }
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();
+}
+
+__global__ void __launch_bounds__(256) k_dense_to_band_tiled(const double *__restrict__ A, long long lda, long long n,
+                                                             int kl, int ku, double *__restrict__ AB, long long ldab,
+                                                             int T) {
+  extern __shared__ double tile[];  // T * ldab, tile[c*ldab + r] = AB(r, j0+c)
+  const long long j0 = (long long)blockIdx.x * T;
+  const int tcols = (int)min((long long)T, n - j0);
+  const long long tsize = (long long)tcols * ldab;
+  fill_band_tile(A, lda, n, kl, ku, j0, tcols, ldab, tile);
   double *out = AB + j0 * ldab;
   for (long long e = threadIdx.x; e < tsize; e += blockDim.x) out[e] = tile[e];
 }
@@ -67,21 +85,10 @@ __global__ void __launch_bounds__(256) k_decide_convert_tiled(const double *__re
   if (blockIdx.x == 0 && threadIdx.x == 0) *d_status = banded ? BANDLU_OK : BANDLU_NOT_BANDED;
   if (!banded) return;  // whole block
   extern __shared__ double tile[];
-  const long long kv = kl + ku;
   const long long j0 = (long long)blockIdx.x * T;
   const int tcols = (int)min((long long)T, n - j0);
   const long long tsize = (long long)tcols * ldab;
-  for (long long e = threadIdx.x; e < tsize; e += blockDim.x) tile[e] = 0.0;
-  __syncthreads();
-  const long long i_lo = max(0ll, j0 - ku);
-  const long long i_hi = min(n - 1, j0 + tcols - 1 + kl);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
-  for (long long i = i_lo + warp; i <= i_hi; i += nwarps) {
-    const long long c_lo = max(j0, i - kl);
-    const long long c_hi = min(min(j0 + tcols - 1, i + ku), n - 1);
-    for (long long c = c_lo + lane; c <= c_hi; c += 32) tile[(c - j0) * ldab + (kv + i - c)] = A[i * lda + c];
-  }
-  __syncthreads();
+  fill_band_tile(A, lda, n, kl, ku, j0, tcols, ldab, tile);
   double *out = AB + j0 * ldab;
   for (long long e = threadIdx.x; e < tsize; e += blockDim.x) out[e] = tile[e];
 }
