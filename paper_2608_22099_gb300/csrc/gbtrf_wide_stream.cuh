@@ -30,7 +30,10 @@
 //    an update CTA has applied panels p_first(b)..b-kHandChain), applies panel
 //    b-r to it as that panel's steps arrive (the pivot row and row j broadcast
 //    inside the CTA, which holds the whole block), and passes the block to CTA
-//    r-1 with one shared-to-shared bulk copy.  While A factors panel p, streamer
+//    r-1: a sender warp moves the rows the panel leaves unchanged as soon as the
+//    block is in and the destination is free (bulk copies of the runs between
+//    the bands), so the group goes straight to the steps, and the group sends
+//    the panel's band rows from registers after the last step.  While A factors panel p, streamer
 //    r applies panel p to block p+r, so each block reaches A with panels up to
 //    p-1 applied, at most one step after A's last step plus one copy.
 //  * The other CTAs (update CTAs) apply panels p_first(b)..b-kHandChain and hand
@@ -59,6 +62,8 @@ struct StreamShared {
   unsigned long long mb_blk[kRing];            // A: block b >= 1 arrived (1 arrival + bytes), event b-1
   unsigned long long mb_afree[kRing];          // streamer 1: A's buffer of block p stored (A's storer), event p
   unsigned long long mb_pub[kRing];            // A: panel p published (publisher), event p
+  unsigned long long mb_dst[kSlots];           // streamer: block b's destination free and its unchanged
+                                               // rows sent (sender), event (b-1) / kSlots
   alignas(16) unsigned long long rhdr[kRecDepth * kNB][2];  // streamer: pivot offset and zero flag of (q, k)
   double lm[32 * CW];  // A: each thread's multiplier of the last step of the panel just factored
 };
@@ -356,7 +361,10 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
       mbar_init(&ss.mb_pub[i], 1);
     }
     for (int i = 0; i < kRecDepth * kNB; ++i) mbar_init(&ss.mb_rec[i], 1);
-    for (int i = 0; i < kSlots; ++i) mbar_init(&ss.mb_in[i], 1);
+    for (int i = 0; i < kSlots; ++i) {
+      mbar_init(&ss.mb_in[i], 1);
+      mbar_init(&ss.mb_dst[i], 1);
+    }
     sh.info = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -425,10 +433,24 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
     }
   } else if (blockIdx.x < kChainCTAs) {
     const int r = blockIdx.x;  // streamer r: panel b-r to block b, then block b to CTA r-1
+    const int ld = (int)g.ldab;
+    const int boff = g.kv - kNB * r;  // band position of row 4(b-r), column 0
+    // where block b goes: A's buffer (which held block b-3: its storer must be done), or
+    // streamer r-1's slot (which held block b-kSlots: A must have factored it)
+    auto dest = [&](int b, unsigned &dst, unsigned &dbar) {
+      if (r == 1) {
+        dst = cl_map(buf(b), 0);
+        dbar = cl_map(&ss.mb_blk[(b - 1) % kRing], 0);
+      } else {
+        dst = cl_map(sbuf(b), r - 1);
+        dbar = cl_map(&ss.mb_in[(b - 1) % kSlots], r - 1);
+      }
+    };
+    auto applies = [&](int b) { return b - r >= 0 && b - r >= p_first(g, b); };
+    const int sender = r < kStreamers ? kCW : kCW + 1;
     if (warp < kCW) {
       int bpar = 0;
       const int i = tid;
-      const int ld = (int)g.ldab;
       for (int b = 1; b < g.npan; ++b) {
         const int slot = (b - 1) % kSlots;
         const int c0b = b * kNB, ncb = min(kNB, g.n - c0b);
@@ -440,33 +462,98 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) break;
         }
         const int q = b - r;
-        const bool apply = q >= 0 && q >= p_first(g, b);  // uniform
+        const bool apply = applies(b);  // uniform
         double *bx = sbuf(b);
-        // where the block goes: A's buffer (which held block b-3: its storer must be done), or
-        // streamer r-1's slot (which held block b-kSlots: A must have factored it)
         unsigned dst, dbar;
+        dest(b, dst, dbar);
+        double w[kNB];  // this thread's row of panel q's band in the block
+        if (q >= 0) {
+          // panel q as its steps stream from A (streamer 1 leaves the last one to A); the
+          // records are taken whether or not the panel reaches this block
+          const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
+          const int nsteps = r == 1 ? ncq - 1 : ncq;
+          const int row = c0q + i;
+          const bool mine = i < g.kl + kNB && row < g.n;
+#pragma unroll
+          for (int d = 0; d < kNB; ++d) {
+            const int pos = boff + i - d;
+            w[d] = (apply && i < g.kl + kNB && d < ncb && pos >= 0 && pos < ld) ? bx[d * ld + pos] : 0.0;
+          }
+          bool ok = true;
+#pragma unroll
+          for (int k = 0; k < kNB; ++k) {
+            if (k >= nsteps) break;  // uniform
+            const int sl = rslot(q, k);
+            // the last streamer opens its own phases; the others' forwarder has opened them
+            if (r == kStreamers && tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
+            unsigned long long *mb = &ss.mb_rec[sl];
+            const unsigned par = ring_parity(q, kRecDepth);
+            if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) {
+              ok = false;
+              break;
+            }
+            if (apply && !ss.rhdr[sl][1]) {  // uniform
+              const double l = recs[(size_t)sl * kCT + i];
+              const int pk = (int)ss.rhdr[sl][0];
+              const int km = min(g.kl, g.n - 1 - (c0q + k));
+              double wm[kNB];
+#pragma unroll
+              for (int d = 0; d < kNB; ++d) wm[d] = w[d];
+              apply_step_regs<CW>(g, wm, i, k, km, pk, l, sh.bc[1], kBarB, bpar);
+              if (mine) {
+#pragma unroll
+                for (int d = 0; d < kNB; ++d) w[d] = wm[d];
+              }
+            }
+          }
+          if (!ok) break;
+        }
+        {
+          // the destination is free (the sender has seen it) and the unchanged rows are on their way
+          unsigned long long *mb = &ss.mb_dst[slot];
+          const unsigned par = ring_parity(b - 1, kSlots);
+          if (!grp_wait([&] { return mbar_try_wait(mb, par); }, kBarB)) break;
+        }
+        if (q >= 0) {
+          // the band: one value per (row, column), from the row's thread
+          if (apply && i < g.kl + kNB) {
+#pragma unroll
+            for (int d = 0; d < kNB; ++d) {
+              const int pos = boff + i - d;
+              if (d < ncb && pos >= 0 && pos < ld) st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(w[d]), dbar);
+            }
+          }
+        }
+      }
+    } else if (warp == sender) {
+      // ---------------- sender: the rows panel b-r leaves unchanged, as soon as they can go ----------------
+      // Panel b-r's rows of block b (band positions boff-d .. boff+kl+3-d of column d) change in
+      // the group; every other value is final and goes now.  Between the bands the block is
+      // ncb+1 runs (a column's tail and the next column's head are contiguous): each a bulk copy
+      // between 16-byte boundaries (lane 0), the at most one value cut off at each end as an
+      // 8-byte st.async (lanes 1 and 2).  Then one arrival tells the group it may send the band.
+      for (int b = 1; b < g.npan; ++b) {
+        const int slot = (b - 1) % kSlots;
+        const int ncb = min(kNB, g.n - b * kNB);
+        {
+          unsigned long long *mb = &ss.mb_in[slot];
+          const unsigned par = ring_parity(b - 1, kSlots);
+          if (!io_wait_all([&] { return cl_try_wait(mb, par); }, err)) break;
+        }
         if (r == 1) {
           if (b >= 3) {
             unsigned long long *mb = &ss.mb_afree[(b - 3) % kRing];
             const unsigned par = ring_parity(b - 3, kRing);
-            if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) break;
+            if (!io_wait_all([&] { return cl_try_wait(mb, par); }, err)) break;
           }
-          dst = cl_map(buf(b), 0);
-          dbar = cl_map(&ss.mb_blk[(b - 1) % kRing], 0);
-        } else {
-          if (b - kSlots >= 1) {
-            const int *f = panel_ready + (b - kSlots);
-            if (!grp_wait([&] { return ld_acquire(f) != 0; }, kBarB)) break;
-          }
-          dst = cl_map(sbuf(b), r - 1);
-          dbar = cl_map(&ss.mb_in[(b - 1) % kSlots], r - 1);
+        } else if (b - kSlots >= 1) {
+          const int *f = panel_ready + (b - kSlots);
+          if (!io_wait_all([&] { return ld_acquire(f) != 0; }, err)) break;
         }
-        // panel q's rows of the block (band positions kv-4r-d .. kv-4r+kl+3-d of column d) change
-        // here; every other value is final for this move and goes now.  Between the bands the
-        // block is ncb+1 runs (a column's tail and the next column's head are contiguous); run
-        // j goes from warp j: a bulk copy between 16-byte boundaries (lane 0), the at most one
-        // value cut off at each end as an 8-byte st.async (lanes 1 and 2)
-        const int boff = g.kv - kNB * r;  // band position of row 4q, column 0
+        const bool apply = applies(b);
+        const double *bx = sbuf(b);
+        unsigned dst, dbar;
+        dest(b, dst, dbar);
         auto band = [&](int d, int &lo, int &hi) {  // band of column d, [lo, hi]; lo > hi: none
           lo = ld;
           hi = ld - 1;
@@ -478,7 +565,8 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
             }
           }
         };
-        for (int j = warp; j <= ncb; j += kCW) {
+        if (lane == 0) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        for (int j = 0; j <= ncb; ++j) {
           int e0, e1;  // element range of run j
           if (j == 0) {
             int lo, hi;
@@ -514,63 +602,18 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
             }
           }
         }
-        if (q >= 0) {
-          // panel q as its steps stream from A (streamer 1 leaves the last one to A); the
-          // records are taken whether or not the panel reaches this block
-          const int c0q = q * kNB, ncq = min(kNB, g.n - c0q);
-          const int nsteps = r == 1 ? ncq - 1 : ncq;
-          const int row = c0q + i;
-          const bool mine = i < g.kl + kNB && row < g.n;
-          double w[kNB];
-#pragma unroll
-          for (int d = 0; d < kNB; ++d) {
-            const int pos = boff + i - d;
-            w[d] = (apply && i < g.kl + kNB && d < ncb && pos >= 0 && pos < ld) ? bx[d * ld + pos] : 0.0;
-          }
-          bool ok = true;
-#pragma unroll
-          for (int k = 0; k < kNB; ++k) {
-            if (k >= nsteps) break;  // uniform
-            const int sl = rslot(q, k);
-            if (tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
-            unsigned long long *mb = &ss.mb_rec[sl];
-            const unsigned par = ring_parity(q, kRecDepth);
-            if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) {
-              ok = false;
-              break;
-            }
-            if (apply && !ss.rhdr[sl][1]) {  // uniform
-              const double l = recs[(size_t)sl * kCT + i];
-              const int pk = (int)ss.rhdr[sl][0];
-              const int km = min(g.kl, g.n - 1 - (c0q + k));
-              double wm[kNB];
-#pragma unroll
-              for (int d = 0; d < kNB; ++d) wm[d] = w[d];
-              apply_step_regs<CW>(g, wm, i, k, km, pk, l, sh.bc[1], kBarB, bpar);
-              if (mine) {
-#pragma unroll
-                for (int d = 0; d < kNB; ++d) w[d] = wm[d];
-              }
-            }
-          }
-          if (!ok) break;
-          // the band: one value per (row, column), from the row's thread
-          if (apply && i < g.kl + kNB) {
-#pragma unroll
-            for (int d = 0; d < kNB; ++d) {
-              const int pos = boff + i - d;
-              if (d < ncb && pos >= 0 && pos < ld) st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(w[d]), dbar);
-            }
-          }
-        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ss.mb_dst[slot]);
       }
     } else if (warp == kCW + 1 && r < kStreamers) {
       // ---------------- forwarder: panel q's step records on to streamer r+1 ----------------
       // This streamer takes panel q iff block q+r exists, streamer r+1 iff block q+r+1 does.
-      // The group's thread 0 opens each step's phase (expect_tx) before its wait, except for
-      // the step streamer 1 leaves to A: that one is opened here.  Slot (q, k) held (q-5, k),
-      // whose phase this warp has seen complete; streamer r+1 has read its own copy of
-      // (q-5, k) before A can send (q, k), so both slots are free.
+      // This warp opens every step's phase (expect_tx) itself, so a phase completes as soon as
+      // its records land, however far behind the group is, and the records move on at once.
+      // Slot (q, k) held (q-5, k), whose phase this warp has seen complete; this streamer's
+      // group and streamer r+1 have read (q-5, k) before A can send (q, k) (block q+5 has
+      // passed through both), so both slots are free and the group's wait on (q-5, k)'s
+      // parity cannot be confused with (q, k)'s.
       const unsigned rbytes = (unsigned)(kCT * 8);
       bool ok = true;
       for (int q = 0; ok && q + r < g.npan; ++q) {
@@ -579,7 +622,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
         for (int k = 0; k < ncq; ++k) {
           const int sl = rslot(q, k);
           unsigned long long *mb = &ss.mb_rec[sl];
-          if (r == 1 && k == ncq - 1 && lane == 0) mbar_expect_tx_local(mb, rbytes + 16u);
+          if (lane == 0) mbar_expect_tx_local(mb, rbytes + 16u);
           const unsigned par = ring_parity(q, kRecDepth);
           if (!io_wait_all([&] { return cl_try_wait(mb, par); }, err)) {
             ok = false;
