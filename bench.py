@@ -20,6 +20,7 @@ oracle's times on this host (single-threaded and with OpenMP).
   python bench.py --workload NAME [--steps K]     per-stage report of a named workload
   python bench.py --custom N KL KU [BATCH]        the same report for a synthetic shape
   python bench.py --sweep                         the paper's experiments A-C on this GPU
+  python bench.py --trace [--custom N KL KU]      timeline of the wide-band chain kernel (traced build)
 """
 from __future__ import annotations
 
@@ -1063,6 +1064,94 @@ def run_sweep(args):
         del A, AB
 
 
+def run_trace(args):
+    """Timeline of the wide-band chain kernel from the traced build (include/bandlu_trace.h):
+    one factorisation of the workload's band (after two untimed ones), the global timer at
+    every panel boundary and wait of the panel CTA, streamers 1 and 2 and the last streamer's
+    loader, summarised over the panels away from both ends.  One JSON line."""
+    os.environ["BANDLU_TRACE"] = "1"  # before the library is loaded
+    import torch
+
+    from paper_2608_22099_gb300 import bandlu
+    from paper_2608_22099_gb300.workloads import WORKLOADS, Workload, make_workload
+
+    if args.custom:
+        cn, ckl, cku = args.custom[:3]
+        w = Workload(f"custom_n{cn}_kl{ckl}_ku{cku}", cn, ckl, cku, "uniform", 0.0, 7)
+    else:
+        w = WORKLOADS[args.workload]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    bandlu.load()
+    cap = bandlu.bandlu_trace_capacity()
+    if cap <= 0:
+        raise RuntimeError("the traced library was not loaded")
+    n, kl, ku, ldab = w.n, w.kl, w.ku, w.ldab
+    kern = gbtrf_kernel(n, kl, ku)
+    A = make_workload(w, device=dev)
+    AB0 = torch.zeros((n, ldab), dtype=torch.float64, device=dev)
+    stream = torch.cuda.current_stream()
+    bandlu.check(bandlu.dense_to_band(A, n, n, kl, ku, AB0, ldab, stream), "convert")
+    del A
+    AB = torch.empty_like(AB0)
+    ipiv = torch.zeros(n, dtype=torch.int32, device=dev)
+    info = torch.zeros(1, dtype=torch.int32, device=dev)
+    times = []
+    for rep in range(3):
+        AB.copy_(AB0)
+        if rep == 2:
+            bandlu.check(bandlu.bandlu_trace_clear(), "trace_clear")
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        bandlu.check(bandlu.gbtrf(n, kl, ku, AB, ldab, ipiv, info, stream), "gbtrf")
+        b.record(stream)
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(b))
+    T = np.zeros(4 * cap * 16, dtype=np.uint64)
+    bandlu.check(bandlu.bandlu_trace_read(T, T.size), "trace_read")
+    T = T.reshape(4, cap, 16).astype(np.int64)
+    npan = (n + 3) // 4
+    lo, hi = min(64, npan // 4), min(cap, npan) - min(64, npan // 4)
+    out = {"mode": "trace", "workload": w.name, "kernel": kern, "n": n, "kl": kl, "ku": ku,
+           "gbtrf_ms_traced_run": times[2],
+           "panels_summarised": [lo, hi], "unit": "ns"}
+    if kern != "k_gbtrf_wide_chain" or hi - lo < 8 or not T[0, lo:hi, 0].all():
+        out["note"] = "no chain-kernel timeline for this band"
+        print(json.dumps(out))
+        return
+
+    def st(x):
+        x = np.asarray(x, dtype=np.float64)
+        return {"median": float(np.median(x)), "mean": float(x.mean()), "p90": float(np.percentile(x, 90))}
+    A0, S1, S2, L = T[0], T[1], T[2], T[3]
+    q = np.arange(lo, hi)
+    out["panel_cta"] = {
+        "period": st(A0[q + 1, 0] - A0[q, 0]),
+        "factor_to_step2_records_sent": st(A0[q, 1] - A0[q, 0]),
+        "step2_records_sent_to_panel_done": st(A0[q, 2] - A0[q, 1]),
+        "wait_for_next_block": st(A0[q, 3] - A0[q, 2]),
+        "block_in_to_next_panel_start": st(A0[q + 1, 0] - A0[q, 3]),
+    }
+    # streamer 1 applies panel q's steps 0..2 to block q+1; its last records are step 2's
+    out["streamer1"] = {
+        "block_in_to_first_records": st(S1[q, 1] - S1[q, 0]),
+        "last_records_wait_starts_after_sent": st(S1[q, 2] - A0[q, 1]),
+        "last_records_seen_after_sent": st(S1[q, 3] - A0[q, 1]),
+        "last_step_and_band_send": st(S1[q, 4] - S1[q, 3]),
+        "band_sent_to_panel_cta_has_block": st(A0[q, 3] - S1[q, 4]),
+    }
+    out["streamer2"] = {
+        "block_in_to_first_records": st(S2[q, 1] - S2[q, 0]),
+        "last_records_seen_after_panel_cta_done": st(S2[q, 3] - A0[q, 2]),
+        "band_sent_to_streamer1_block_in": st(S1[q + 1, 0] - S2[q, 4]),
+    }
+    bq = q[L[q, 0] > 0]
+    out["loader_wait_for_hand_over"] = st(L[bq, 1] - L[bq, 0]) if bq.size else None
+    print(json.dumps(out))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -1074,6 +1163,8 @@ def main():
                     help="workload name (default: the n=32768, kl=ku=256 matrix); others for per-workload reports")
     ap.add_argument("--sweep", action="store_true", help="the paper's experiments A-C (speedup / slowdown in N)")
     ap.add_argument("--peaks", action="store_true", help="FP64 FMA / DMMA and HBM read microbenchmarks")
+    ap.add_argument("--trace", action="store_true",
+                    help="timeline of the wide-band chain kernel from the traced build (bandlu_trace.h)")
     ap.add_argument("--custom", type=int, nargs="+", metavar="N KL KU [BATCH]",
                     help="per-stage report of a synthetic uniform[-1,1] band of this shape (batched if BATCH > 0)")
     args = ap.parse_args()
@@ -1081,6 +1172,8 @@ def main():
         ap.error("--custom takes N KL KU [BATCH]")
     if args.impl == "reference":
         run_reference(args)
+    elif args.trace:
+        run_trace(args)
     elif args.peaks:
         run_peaks(args)
     elif args.sweep:

@@ -41,10 +41,12 @@ def load():
         # BANDLU_CHECKED=1 selects the checked build (bounded inter-warp waits) for
         # development runs; the default is the production library.
         checked = os.environ.get("BANDLU_CHECKED", "") == "1"
-        path = _build.CHECKED_LIB if checked else _build.LIB
+        # BANDLU_TRACE=1 selects the traced build (timeline of the wide-band chain kernel)
+        trace = not checked and os.environ.get("BANDLU_TRACE", "") == "1"
+        path = _build.CHECKED_LIB if checked else (_build.TRACE_LIB if trace else _build.LIB)
         if not _build.up_to_date(path):
             try:
-                path = _build.build(checked=checked)
+                path = _build.build(checked=checked, trace=trace)
             except Exception as e:  # noqa: BLE001 - re-raised with context
                 raise BandLUError(f"the CUDA library could not be built: {e}") from e
         if not os.path.exists(path):
@@ -72,6 +74,12 @@ def load():
                   "detect_bandwidth_cm", "dense_to_band_cm", "dispatch_lu_cm", "diag_solve", "bandlu_classify",
                   "dispatch_backslash"):
             getattr(lib, f).restype = ctypes.c_int
+        lib.bandlu_trace_capacity.argtypes = []
+        lib.bandlu_trace_capacity.restype = ctypes.c_int
+        lib.bandlu_trace_read.argtypes = [vp, i64]
+        lib.bandlu_trace_read.restype = ctypes.c_int
+        lib.bandlu_trace_clear.argtypes = []
+        lib.bandlu_trace_clear.restype = ctypes.c_int
         lib.bandlu_selftest_rcp_host.argtypes = [vp, vp, i64]
         lib.bandlu_selftest_rcp_host.restype = None
         lib.bandlu_selftest_rcp_device.argtypes = [vp, vp, i64, i32, vp]
@@ -211,6 +219,21 @@ def dispatch_lu_batched(A, n: int, lda: int, strideA: int, batch: int, AB, ldab:
     return load().dispatch_lu_batched(_ptr(A), n, lda, strideA, batch, _ptr(AB), ldab, strideAB, _ptr(ipiv),
                                       strideP, _ptr(d_kl), _ptr(d_ku), _ptr(d_info), _ptr(d_status),
                                       _stream(stream))
+
+
+def bandlu_trace_capacity() -> int:
+    """Panels the traced build records per role (0 in the production build)."""
+    return load().bandlu_trace_capacity()
+
+
+def bandlu_trace_read(host, count: int) -> int:
+    """Copies the first `count` words of the chain kernel's timeline to `host` (host buffer)."""
+    return load().bandlu_trace_read(_ptr_host(host), count)
+
+
+def bandlu_trace_clear() -> int:
+    """Zeroes the timeline (traced build)."""
+    return load().bandlu_trace_clear()
 
 
 def bandlu_selftest_rcp_host(x, y, n: int) -> None:

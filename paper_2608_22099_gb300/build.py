@@ -23,6 +23,10 @@ LIB = os.path.join(BUILD, "libbandlu.so")
 # mbarrier waits (a protocol slip ends a kernel with an error status instead of
 # a hang).  Never the library the product path loads.
 CHECKED_LIB = os.path.join(BUILD, "libbandlu_checked.so")
+# Traced variant for development and profiling: the wide-band chain kernel records the global
+# timer at its panel boundaries and waits (include/bandlu_trace.h).  Never the library the
+# product path loads.
+TRACE_LIB = os.path.join(BUILD, "libbandlu_trace.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
@@ -52,16 +56,17 @@ def up_to_date(lib: str = LIB) -> bool:
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | None = None,
-          checked: bool = False) -> str:
-    """Compile and link the library (or its checked variant); returns its path.
+          checked: bool = False, trace: bool = False) -> str:
+    """Compile and link the library (or its checked or traced variant); returns its path.
     Raises on a compiler error."""
-    lib = CHECKED_LIB if checked else LIB
+    lib = CHECKED_LIB if checked else (TRACE_LIB if trace else LIB)
     if not force and up_to_date(lib):
         return lib
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
-    flags = NVCC_FLAGS + list(extra_flags or []) + (["-DBANDLU_BOUNDED_SYNC"] if checked else [])
-    suffix = ".checked.o" if checked else ".o"
+    flags = NVCC_FLAGS + list(extra_flags or []) + (["-DBANDLU_BOUNDED_SYNC"] if checked else []) + \
+        (["-DBANDLU_TRACE"] if trace else [])
+    suffix = ".checked.o" if checked else (".trace.o" if trace else ".o")
 
     def compile_one(src: str) -> str:
         obj = os.path.join(BUILD, os.path.basename(src)[:-3] + suffix)
@@ -87,4 +92,4 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
 if __name__ == "__main__":
     print(build(force="--force" in sys.argv, verbose="-v" in sys.argv,
                 extra_flags=["-Xptxas", "-v"] if "--ptxas-v" in sys.argv else None,
-                checked="--checked" in sys.argv))
+                checked="--checked" in sys.argv, trace="--trace" in sys.argv))

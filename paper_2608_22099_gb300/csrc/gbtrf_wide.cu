@@ -54,6 +54,7 @@
 #include <mutex>
 #include <tuple>
 
+#include "bandlu_trace.h"
 #include "common.cuh"
 #include "rcp.cuh"
 #include "sync.cuh"
@@ -1369,3 +1370,41 @@ int launch_gbtrf_wide_deferred(const WideDeferred &wd, int64_t n, double *AB, in
 }
 
 }  // namespace bandlu
+
+// ---- timeline of the traced build (include/bandlu_trace.h) ----
+extern "C" {
+
+int bandlu_trace_capacity(void) {
+#ifdef BANDLU_TRACE
+  return bandlu::kTrPanels;
+#else
+  return 0;
+#endif
+}
+
+int bandlu_trace_read(uint64_t *host, int64_t count) {
+#ifdef BANDLU_TRACE
+  if (host == nullptr) return -1;
+  if (count < 0 || count > 4ll * bandlu::kTrPanels * bandlu::kTrSlots) return -2;
+  if (count == 0) return BANDLU_OK;
+  return cudaMemcpyFromSymbol(host, bandlu::g_chain_trace, (size_t)count * sizeof(uint64_t)) == cudaSuccess
+             ? BANDLU_OK
+             : BANDLU_ERR_CUDA;
+#else
+  (void)host;
+  (void)count;
+  return BANDLU_ERR_CUDA;
+#endif
+}
+
+int bandlu_trace_clear(void) {
+#ifdef BANDLU_TRACE
+  void *p = nullptr;
+  if (cudaGetSymbolAddress(&p, bandlu::g_chain_trace) != cudaSuccess) return BANDLU_ERR_CUDA;
+  return cudaMemset(p, 0, sizeof(bandlu::g_chain_trace)) == cudaSuccess ? BANDLU_OK : BANDLU_ERR_CUDA;
+#else
+  return BANDLU_ERR_CUDA;
+#endif
+}
+
+}  // extern "C"

@@ -48,6 +48,28 @@
 // (b-kSlots) A has already factored (panel_ready).  Every wait is bounded.
 #pragma once
 
+// Timeline of the traced build (include/bandlu_trace.h): the global timer at panel
+// boundaries and waits; nothing in the production build.
+constexpr int kTrPanels = 8192, kTrSlots = 16;
+#ifdef BANDLU_TRACE
+__device__ unsigned long long g_chain_trace[4][kTrPanels][kTrSlots];
+__device__ __forceinline__ void tr_stamp(int role, int q, int slot) {
+  if (q >= 0 && q < kTrPanels) {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    g_chain_trace[role][q][slot] = t;
+  }
+}
+#define TR_STAMP(cond, role, q, slot) \
+  do {                                \
+    if (cond) tr_stamp(role, q, slot); \
+  } while (0)
+#else
+#define TR_STAMP(cond, role, q, slot) \
+  do {                                \
+  } while (0)
+#endif
+
 constexpr int kStreamers = 4;                    // streamer CTAs after A
 constexpr int kChainCTAs = kStreamers + 1;       // cluster size
 constexpr int kRecDepth = kStreamers + 1;        // panels of step records per streamer
@@ -270,6 +292,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
         st_async_v2(rt.hdr + (unsigned)k * 16u, (unsigned long long)(unsigned)p_off, zero ? 1ull : 0ull,
                     rt.bar + (unsigned)k * 8u);
     }
+    TR_STAMP(k == 2 && tid == 0, 0, p, 1);
   }
   if (mine) {
 #pragma unroll
@@ -390,6 +413,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
         rt.hdr = cl_map(&ss.rhdr[rslot(p, 0)][0], 1);
         rt.bar = cl_map(&ss.mb_rec[rslot(p, 0)], 1);
         rt.send = p + 1 < g.npan;  // streamer 1 applies panel p to block p+1
+        TR_STAMP(tid == 0, 0, p, 0);
         factor_panel_stream<CW>(g, buf(p), p, sh, bpar, info, rt, AB, ipiv, ss.lm, p > 0);
         if (tid == 0) {
           sh.info = info;
@@ -398,10 +422,12 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
         }
         bar_compute<CW>();
         if (tid == 0) mbar_arrive(&sh.mb_done[p % kRing]);  // the storer
+        TR_STAMP(tid == 0, 0, p, 2);
         if (p + 1 < g.npan) {
           unsigned long long *mb = &ss.mb_blk[p % kRing];
           const unsigned par = ring_parity(p, kRing);
           if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarA)) break;
+          TR_STAMP(tid == 0, 0, p, 3);
           // block p+1 holds panel p's steps but the last, which the next factor_panel_stream applies
         }
       }
@@ -461,6 +487,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           const unsigned par = ring_parity(b - 1, kSlots);
           if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) break;
         }
+        TR_STAMP(r <= 2 && tid == 0, r, b - r, 0);
         const int q = b - r;
         const bool apply = applies(b);  // uniform
         double *bx = sbuf(b);
@@ -488,10 +515,13 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
             if (r == kStreamers && tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
             unsigned long long *mb = &ss.mb_rec[sl];
             const unsigned par = ring_parity(q, kRecDepth);
+            TR_STAMP(r <= 2 && tid == 0 && k == nsteps - 1, r, q, 2);
             if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) {
               ok = false;
               break;
             }
+            TR_STAMP(r <= 2 && tid == 0 && k == 0, r, q, 1);
+            TR_STAMP(r <= 2 && tid == 0 && k == nsteps - 1, r, q, 3);
             if (apply && !ss.rhdr[sl][1]) {  // uniform
               const double l = recs[(size_t)sl * kCT + i];
               const int pk = (int)ss.rhdr[sl][0];
@@ -523,6 +553,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
               if (d < ncb && pos >= 0 && pos < ld) st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(w[d]), dbar);
             }
           }
+          TR_STAMP(r <= 2 && tid == 0, r, q, 4);
         }
       }
     } else if (warp == sender) {
@@ -657,7 +688,9 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
         unsigned long long *ml = &ss.mb_in[(b - 1) % kSlots];
         if (handed_off_chain(g, b)) {
           const int *f = block_ready + b;
+          TR_STAMP(lane == 0, 3, b, 0);
           if (!io_wait_all([&] { return ld_acquire(f) != 0; }, err)) break;
+          TR_STAMP(lane == 0, 3, b, 1);
           if (g.vec && (b + 1) * kNB <= g.n) {
             if (lane == 0) bulk_prefetch_block(g, AB, dst, b, ml);  // completes the phase itself
             __syncwarp();
