@@ -88,6 +88,10 @@ struct StreamShared {
                                                // rows sent (sender), event (b-1) / kSlots
   alignas(16) unsigned long long rhdr[kRecDepth * kNB][2];  // streamer: pivot offset and zero flag of (q, k)
   double lm[32 * CW];  // A: each thread's multiplier of the last step of the panel just factored
+  // streamer: every thread's row of the block before a step (the step's pivot row and row j
+  // are read from here), by step parity
+  double rows[2][32 * CW][kNB];
+  unsigned rmask[2][32 * CW];
 };
 
 __device__ __forceinline__ unsigned long long dbl_bits_w(double x) {
@@ -341,6 +345,28 @@ __device__ __forceinline__ void apply_step_regs(const Geo &g, double (&w)[kNB], 
   }
 }
 
+// One step k of panel q on a streamer's rows (registers w), after the step's barrier:
+// the pivot row and row j come from the rows every thread published before it.
+template <int CW>
+__device__ __forceinline__ void apply_step_published(double (&w)[kNB], int i, int k, int km, int p, double l,
+                                                     const double (*rows)[kNB], const unsigned *rmask) {
+  double u[kNB];
+#pragma unroll
+  for (int d = 0; d < kNB; ++d) u[d] = rows[k + p][d];
+  const unsigned um = rmask[k + p];
+  if (i == k) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = u[d];
+  } else if (p != 0 && i == k + p) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = rows[k][d];
+  }
+  if (i > k && i <= k + km) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = upd(l, u[d], w[d], (um >> d) & 1u);
+  }
+}
+
 // Blocks b >= kHandChain pass through an update CTA, which applies panels
 // p_first(b)..b-kHandChain.
 __device__ __forceinline__ bool handed_off_chain(const Geo &g, int b) {
@@ -511,6 +537,13 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           for (int k = 0; k < kNB; ++k) {
             if (k >= nsteps) break;  // uniform
             const int sl = rslot(q, k);
+            // this thread's row as it stands, for the step's pivot row and row j; the wait's
+            // barrier below makes every row visible (slot bpar was last read two steps ago)
+            const int sb = bpar;
+            bpar ^= 1;
+#pragma unroll
+            for (int d = 0; d < kNB; ++d) ss.rows[sb][i][d] = w[d];
+            ss.rmask[sb][i] = nz_mask(w);
             // the last streamer opens its own phases; the others' forwarder has opened them
             if (r == kStreamers && tid == 0) mbar_expect_tx_local(&ss.mb_rec[sl], (unsigned)(kCT * 8 + 16));
             unsigned long long *mb = &ss.mb_rec[sl];
@@ -529,7 +562,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
               double wm[kNB];
 #pragma unroll
               for (int d = 0; d < kNB; ++d) wm[d] = w[d];
-              apply_step_regs<CW>(g, wm, i, k, km, pk, l, sh.bc[1], kBarB, bpar);
+              apply_step_published<CW>(wm, i, k, km, pk, l, ss.rows[sb], ss.rmask[sb]);
               if (mine) {
 #pragma unroll
                 for (int d = 0; d < kNB; ++d) w[d] = wm[d];
