@@ -367,6 +367,31 @@ __device__ __forceinline__ void apply_step_published(double (&w)[kNB], int i, in
   }
 }
 
+// The same for a block's last step, handing each column's final value to send(d, x) as soon
+// as it is formed, so the sends overlap the updates of the columns after it.
+template <int CW, class Send>
+__device__ __forceinline__ void apply_step_published_send(double (&w)[kNB], int i, int k, int km, int p, double l,
+                                                          const double (*rows)[kNB], const unsigned *rmask,
+                                                          Send send) {
+  double u[kNB];
+#pragma unroll
+  for (int d = 0; d < kNB; ++d) u[d] = rows[k + p][d];
+  const unsigned um = rmask[k + p];
+  if (i == k) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = u[d];
+  } else if (p != 0 && i == k + p) {
+#pragma unroll
+    for (int d = 0; d < kNB; ++d) w[d] = rows[k][d];
+  }
+  const bool act = i > k && i <= k + km;
+#pragma unroll
+  for (int d = 0; d < kNB; ++d) {
+    if (act) w[d] = upd(l, u[d], w[d], (um >> d) & 1u);
+    send(d, w[d]);
+  }
+}
+
 // Blocks b >= kHandChain pass through an update CTA, which applies panels
 // p_first(b)..b-kHandChain.
 __device__ __forceinline__ bool handed_off_chain(const Geo &g, int b) {
@@ -519,6 +544,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
         double *bx = sbuf(b);
         unsigned dst, dbar;
         dest(b, dst, dbar);
+        bool sent = false;  // the band went out within the last step
         double w[kNB];  // this thread's row of panel q's band in the block
         if (q >= 0) {
           // panel q as its steps stream from A (streamer 1 leaves the last one to A); the
@@ -562,7 +588,25 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
               double wm[kNB];
 #pragma unroll
               for (int d = 0; d < kNB; ++d) wm[d] = w[d];
-              apply_step_published<CW>(wm, i, k, km, pk, l, ss.rows[sb], ss.rmask[sb]);
+              if (k == nsteps - 1) {
+                // the block's last step here: the destination must be free before any band row
+                // goes (the sender's arrival, long since made, is taken first)
+                unsigned long long *md = &ss.mb_dst[slot];
+                const unsigned pard = ring_parity(b - 1, kSlots);
+                if (!grp_wait([&] { return mbar_try_wait(md, pard); }, kBarB)) {
+                  ok = false;
+                  break;
+                }
+                apply_step_published_send<CW>(wm, i, k, km, pk, l, ss.rows[sb], ss.rmask[sb], [&](int d, double x) {
+                  const int pos = boff + i - d;
+                  if (i < g.kl + kNB && d < ncb && pos >= 0 && pos < ld)
+                    st_async_b64(dst + (unsigned)(d * ld + pos) * 8u, dbl_bits_w(x), dbar);
+                });
+                sent = true;
+                TR_STAMP(r <= 2 && tid == 0, r, q, 4);
+              } else {
+                apply_step_published<CW>(wm, i, k, km, pk, l, ss.rows[sb], ss.rmask[sb]);
+              }
               if (mine) {
 #pragma unroll
                 for (int d = 0; d < kNB; ++d) w[d] = wm[d];
@@ -571,13 +615,13 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
           }
           if (!ok) break;
         }
-        {
+        if (!sent) {
           // the destination is free (the sender has seen it) and the unchanged rows are on their way
           unsigned long long *mb = &ss.mb_dst[slot];
           const unsigned par = ring_parity(b - 1, kSlots);
           if (!grp_wait([&] { return mbar_try_wait(mb, par); }, kBarB)) break;
         }
-        if (q >= 0) {
+        if (q >= 0 && !sent) {
           // the band: one value per (row, column), from the row's thread
           if (apply && i < g.kl + kNB) {
 #pragma unroll
