@@ -575,7 +575,12 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
             unsigned long long *mb = &ss.mb_rec[sl];
             const unsigned par = ring_parity(q, kRecDepth);
             TR_STAMP(r <= 2 && tid == 0 && k == nsteps - 1, r, q, 2);
-            if (!grp_wait([&] { return cl_try_wait(mb, par); }, kBarB)) {
+            // the block's last step also takes the sender's arrival (destination free), made
+            // long before, in the same wait
+            unsigned long long *md = &ss.mb_dst[slot];
+            const unsigned pard = ring_parity(b - 1, kSlots);
+            const bool lastk = k == nsteps - 1;
+            if (!grp_wait([&] { return cl_try_wait(mb, par) && (!lastk || mbar_try_wait(md, pard)); }, kBarB)) {
               ok = false;
               break;
             }
@@ -588,15 +593,8 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
               double wm[kNB];
 #pragma unroll
               for (int d = 0; d < kNB; ++d) wm[d] = w[d];
-              if (k == nsteps - 1) {
-                // the block's last step here: the destination must be free before any band row
-                // goes (the sender's arrival, long since made, is taken first)
-                unsigned long long *md = &ss.mb_dst[slot];
-                const unsigned pard = ring_parity(b - 1, kSlots);
-                if (!grp_wait([&] { return mbar_try_wait(md, pard); }, kBarB)) {
-                  ok = false;
-                  break;
-                }
+              if (lastk) {
+                // the block's last step here (the destination is free: taken in the wait above)
                 apply_step_published_send<CW>(wm, i, k, km, pk, l, ss.rows[sb], ss.rmask[sb], [&](int d, double x) {
                   const int pos = boff + i - d;
                   if (i < g.kl + kNB && d < ncb && pos >= 0 && pos < ld)
