@@ -286,10 +286,6 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
         pum = um;
       }
     }
-    // column k is final now (later interchanges touch columns k+1.. only): what the update
-    // CTAs read of it, the diagonal and the multipliers (band rows kv..kv+kl), goes straight
-    // into AB, so the publisher only has to release it once the group has arrived
-    if (mine && i >= k && i - k <= g.kl) abp[k * ldab + g.kv + i - k] = v[k];
     if (rt.send) {  // uniform; streamer 1 passes every step on, and applies all but the last
       st_async_b64(rt.rec + (unsigned)(k * kCT + tid) * 8u, dbl_bits_w(lsend), rt.bar + (unsigned)k * 8u);
       if (tid == 0)
@@ -298,10 +294,17 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
     }
     TR_STAMP(k == 2 && tid == 0, 0, p, 1);
   }
+  // every column is final now (an interchange touches the columns from its own on): what the
+  // update CTAs read, the diagonals and the multipliers (band rows kv..kv+kl), goes straight
+  // into AB, so the publisher only has to release it once every warp has arrived
   if (mine) {
 #pragma unroll
-    for (int k = 0; k < kNB; ++k)
-      if (k < nc && i - k <= g.kl) blk[k * ldab + g.kv + i - k] = v[k];
+    for (int k = 0; k < kNB; ++k) {
+      if (k < nc && i - k <= g.kl) {
+        blk[k * ldab + g.kv + i - k] = v[k];
+        if (i >= k) abp[k * ldab + g.kv + i - k] = v[k];
+      }
+    }
   }
   lm[tid] = lastl;  // read by panel p+1 after the group's next barrier
   if (tid == 0) {
@@ -429,7 +432,7 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
 
   if (tid == 0) {
     for (int i = 0; i < kRing; ++i) {
-      mbar_init(&sh.mb_done[i], 1);
+      mbar_init(&sh.mb_done[i], kCW);  // one arrival per warp of group A
       mbar_init(&ss.mb_blk[i], 1);
       mbar_init(&ss.mb_afree[i], 1);
       mbar_init(&ss.mb_pub[i], 1);
@@ -471,8 +474,11 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
 #pragma unroll
           for (int k = 0; k < kNB; ++k) sh.pvr[p % kRing][k] = sh.pk[p & 1][k];
         }
-        bar_compute<CW>();
-        if (tid == 0) mbar_arrive(&sh.mb_done[p % kRing]);  // the storer
+        // the publisher and the storer: each warp arrives once its stores are issued (the
+        // arrival releases them); the next panel's reads of lm and sh.pk are ordered by the
+        // barrier of the wait for block p+1
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh.mb_done[p % kRing]);
         TR_STAMP(tid == 0, 0, p, 2);
         if (p + 1 < g.npan) {
           unsigned long long *mb = &ss.mb_blk[p % kRing];
