@@ -1134,6 +1134,10 @@ def run_trace(args):
         "wait_for_next_block": st(A0[q, 3] - A0[q, 2]),
         "block_in_to_next_panel_start": st(A0[q + 1, 0] - A0[q, 3]),
     }
+    for k in range(4):
+        out["panel_cta"][f"step{k}_start_to_barrier"] = st(A0[q, 5 + 3 * k] - A0[q, 4 + 3 * k])
+        out["panel_cta"][f"step{k}_barrier_to_records_sent"] = st(A0[q, 6 + 3 * k] - A0[q, 5 + 3 * k])
+    out["panel_cta"]["panel_start_to_step0_start"] = st(A0[q, 4] - A0[q, 0])
     # streamer 1 applies panel q's steps 0..2 to block q+1; its last records are step 2's
     out["streamer1"] = {
         "block_in_to_first_records": st(S1[q, 1] - S1[q, 0]),

@@ -16,7 +16,9 @@
  * streamers (the streamer entry of block b applying panel b-r is q = b-r), and
  * block b for the loader; a later call overwrites what an earlier one wrote.
  *   role 0, panel CTA:    0 panel start, 1 step 2's records sent, 2 panel done,
- *                         3 block q+1's first bytes usable (the wait is over)
+ *                         3 block q+1 usable (the wait is over); for column step
+ *                         k = 0..3: 4+3k step start, 5+3k the step's barrier passed
+ *                         (every warp has published), 6+3k its records sent
  *   roles 1, 2, streamers 1 and 2:
  *                         0 block in, 1 first records seen, 2 wait for the last
  *                         step's records begins, 3 last records seen, 4 band sent

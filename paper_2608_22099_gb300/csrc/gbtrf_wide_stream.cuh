@@ -208,6 +208,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
     const int j = c0 + k, km = min(g.kl, g.n - 1 - j);
     const int s = bpar;
     bpar ^= 1;
+    TR_STAMP(tid == 0, 0, p, 4 + 3 * k);
     const int t = i - k;
     bool myspec;
     const double myr = rcp_rn_fast(v[k], &myspec);
@@ -236,6 +237,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
       for (int d = 0; d < kNB; ++d) sh.row0[s][d] = v[d];
     }
     bar_compute<CW>();
+    TR_STAMP(tid == 0, 0, p, 5 + 3 * k);
     if (k == 0 && wrow && tid == 0) {  // every thread has read row jq above
 #pragma unroll
       for (int d = 0; d < kNB; ++d)
@@ -293,6 +295,7 @@ __device__ void factor_panel_stream(const Geo &g, double *blk, int p, WideShared
                     rt.bar + (unsigned)k * 8u);
     }
     TR_STAMP(k == 2 && tid == 0, 0, p, 1);
+    TR_STAMP(tid == 0, 0, p, 6 + 3 * k);
   }
   // every column is final now (an interchange touches the columns from its own on): what the
   // update CTAs read, the diagonals and the multipliers (band rows kv..kv+kl), goes straight
