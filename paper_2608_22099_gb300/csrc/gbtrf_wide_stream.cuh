@@ -827,8 +827,9 @@ __global__ void __launch_bounds__(32 * (CW + 2), 1)
         apply_panel<CW, 1>(g, blk, b, p, lr, sh.pk[0], sh.zp[0], sh.bc[0], tid, kBarA, bpar);
         bar_compute<CW>();
         if (p == b - kHandChain) {
+          // the block to AB, then the hand-over: the barrier orders every thread's stores before
+          // thread 0's release, which (being cumulative) makes them visible with the flag
           store_block(g, AB, blk, b, tid, kCT);
-          __threadfence();
           bar_compute<CW>();
           if (tid == 0) st_release(block_ready + b, 1);
         }
