@@ -1153,6 +1153,10 @@ def run_trace(args):
     }
     bq = q[L[q, 0] > 0]
     out["loader_wait_for_hand_over"] = st(L[bq, 1] - L[bq, 0]) if bq.size else None
+    # the supply path: panel b-5 done on A -> its update CTA has applied it and handed block b
+    # over (the loader sees the flag)
+    bs = bq[bq >= lo + 5]
+    out["panel_done_to_hand_over_seen"] = st(L[bs, 1] - A0[bs - 5, 2]) if bs.size else None
     print(json.dumps(out))
 
 
