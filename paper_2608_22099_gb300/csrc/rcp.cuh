@@ -9,9 +9,10 @@
 // R = 2^105 - Q*m (no ties are possible: 2^106/m is not an integer for m > 2^52).
 // Q is found as a quotient by approximate reciprocal with remainder correction
 // (Knuth, TAOCP Vol. 2, Sec. 4.3.1): a Newton step on a two-float (double-float)
-// representation of m gives Q within 2^8; one correction Q += (2^105 - Q*m)/m,
-// estimated in single precision from the exact 64-bit remainder, brings Q within
-// one unit; the exact remainder then fixes Q and decides the rounding.
+// representation of m gives Q within 2^9; one correction Q += (2^105 - Q*m)/m,
+// the remainder's high bits times y's 24-bit significand in one integer
+// multiply, brings Q within one unit; the exact remainder then fixes Q and
+// decides the rounding.
 // The result is the IEEE round-to-nearest 1/b, bit for bit.  Zeros, subnormals,
 // infinities, NaN and |b| >= 2^1021 (whose reciprocal is subnormal) go to the
 // ordinary division.
@@ -53,6 +54,16 @@ __host__ __device__ __forceinline__ double bitsd(uint64_t u) {
 #endif
 }
 
+__host__ __device__ __forceinline__ float bitsf(uint32_t u) {
+#ifdef __CUDA_ARCH__
+  return __uint_as_float(u);
+#else
+  float x;
+  std::memcpy(&x, &u, 4);
+  return x;
+#endif
+}
+
 __host__ __device__ __forceinline__ uint32_t fbits(float x) {
 #ifdef __CUDA_ARCH__
   return (uint32_t)__float_as_uint(x);
@@ -75,24 +86,28 @@ __host__ __device__ __forceinline__ double rcp_rn_fast(double b, bool *special) 
   const uint64_t sign = bits & (1ull << 63);
   *special = (E == 0) | (E >= 2045);
   const uint64_t m = frac | (1ull << 52);
-  // M = m / 2^29 = xh + xl/2^29 with xh the 24-bit rounding (exact in single
-  // precision) and |xl| <= 2^28.
-  const uint32_t xh = (uint32_t)(((m >> 28) + 1) >> 1);
-  const int32_t xl = (int32_t)((int64_t)m - ((int64_t)xh << 29));
-  const float xhf = (float)xh, xlf = (float)xl * 0x1p-29f;
+  // M = m / 2^29 = xh + xl/2^29 with xh = floor(M), 2^23 <= xh < 2^24, written straight
+  // into a float's bits (exponent 2^23), and 0 <= xl < 2^29.
+  const uint32_t xh = (uint32_t)(m >> 29);
+  const int32_t xl = (int32_t)(m & ((1ull << 29) - 1));
+  const float xhf = bitsf((150u << 23) | (xh & 0x7fffffu)), xlf = (float)xl * 0x1p-29f;
   // y ~ 1/xh: hardware seed plus one Newton step; then one Newton step for 1/M
-  // carried as the unevaluated pair y + t (relative error below 2^-45).
+  // carried as the unevaluated pair y + t (relative error below 2^-45, plus 2^-47 from
+  // rounding xl to a float).
   const float y0 = rcp_approx_f32(xhf);
   const float y = fmaf(y0, fmaf(-xhf, y0, 1.0f), y0);
   const float e = fmaf(-xlf, y, fmaf(-xhf, y, 1.0f));  // 1 - M*y
   const float t = y * e;
-  // Q = (y + t) * 2^76 ~ 2^105/m within 2^8; y*2^76 is an exact integer (y in [2^-24, 2^-23]).
+  // Q = (y + t) * 2^76 ~ 2^105/m within 2^9; y*2^76 is an exact integer (y in [2^-24, 2^-23]).
   const uint32_t yb = fbits(y);
-  uint64_t Q = (uint64_t)((yb & 0x7fffffu) | 0x800000u) << (int)((yb >> 23) - 74u);
+  const uint32_t ym = (yb & 0x7fffffu) | 0x800000u;  // y = ym * 2^(yexp - 150)
+  const int yexp = (int)(yb >> 23);
+  uint64_t Q = (uint64_t)ym << (yexp - 74);
   Q = (uint64_t)((int64_t)Q + (int64_t)(int32_t)(t * 0x1p76f));
-  // one correction from the exact remainder: 2^105 = 0 mod 2^64 and |R| < 2^62
+  // one correction from the exact remainder (2^105 = 0 mod 2^64 and |R| < 2^62): Q += R/m,
+  // R/m ~ (R >> 31) * y * 2^2 = (R >> 31) * ym / 2^(148 - yexp), floored, within one unit
   int64_t R = (int64_t)(0ull - Q * m);
-  Q = (uint64_t)((int64_t)Q + (int64_t)(int32_t)((float)(int32_t)(R >> 31) * y * 4.0f));
+  Q = (uint64_t)((int64_t)Q + (((int64_t)(int32_t)(R >> 31) * (int64_t)ym) >> (148 - yexp)));
   // now |Q - 2^105/m| < 1.01: the exact remainder fixes Q and decides the rounding
   R = (int64_t)(0ull - Q * m);
   const bool lo = R < 0, hi = R >= (int64_t)m;
