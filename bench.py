@@ -1064,6 +1064,49 @@ def run_sweep(args):
         del A, AB
 
 
+def trace_summary(T: np.ndarray, lo: int, hi: int) -> dict:
+    """Summary of a chain-kernel timeline (roles x entries x slots, include/bandlu_trace.h)
+    over entries [lo, hi): medians, means and 90th percentiles of the intervals between its
+    stamps, in the timer's unit."""
+    def st(x):
+        x = np.asarray(x, dtype=np.float64)
+        return {"median": float(np.median(x)), "mean": float(x.mean()), "p90": float(np.percentile(x, 90))}
+    A0, S1, S2, L = T[0], T[1], T[2], T[3]
+    q = np.arange(lo, hi)
+    out = {}
+    out["panel_cta"] = {
+        "period": st(A0[q + 1, 0] - A0[q, 0]),
+        "factor_to_step2_records_sent": st(A0[q, 1] - A0[q, 0]),
+        "step2_records_sent_to_panel_done": st(A0[q, 2] - A0[q, 1]),
+        "wait_for_next_block": st(A0[q, 3] - A0[q, 2]),
+        "block_in_to_next_panel_start": st(A0[q + 1, 0] - A0[q, 3]),
+    }
+    for k in range(4):
+        out["panel_cta"][f"step{k}_start_to_barrier"] = st(A0[q, 5 + 3 * k] - A0[q, 4 + 3 * k])
+        out["panel_cta"][f"step{k}_barrier_to_records_sent"] = st(A0[q, 6 + 3 * k] - A0[q, 5 + 3 * k])
+    out["panel_cta"]["panel_start_to_step0_start"] = st(A0[q, 4] - A0[q, 0])
+    # streamer 1 applies panel q's steps 0..2 to block q+1; its last records are step 2's
+    out["streamer1"] = {
+        "block_in_to_first_records": st(S1[q, 1] - S1[q, 0]),
+        "last_records_wait_starts_after_sent": st(S1[q, 2] - A0[q, 1]),
+        "last_records_seen_after_sent": st(S1[q, 3] - A0[q, 1]),
+        "last_step_and_band_send": st(S1[q, 4] - S1[q, 3]),
+        "band_sent_to_panel_cta_has_block": st(A0[q, 3] - S1[q, 4]),
+    }
+    out["streamer2"] = {
+        "block_in_to_first_records": st(S2[q, 1] - S2[q, 0]),
+        "last_records_seen_after_panel_cta_done": st(S2[q, 3] - A0[q, 2]),
+        "band_sent_to_streamer1_block_in": st(S1[q + 1, 0] - S2[q, 4]),
+    }
+    bq = q[L[q, 0] > 0]
+    out["loader_wait_for_hand_over"] = st(L[bq, 1] - L[bq, 0]) if bq.size else None
+    # the supply path: panel b-5 done on A -> its update CTA has applied it and handed block b
+    # over (the loader sees the flag)
+    bs = bq[bq >= lo + 5]
+    out["panel_done_to_hand_over_seen"] = st(L[bs, 1] - A0[bs - 5, 2]) if bs.size else None
+    return out
+
+
 def run_trace(args):
     """Timeline of the wide-band chain kernel from the traced build (include/bandlu_trace.h):
     one factorisation of the workload's band (after two untimed ones), the global timer at
@@ -1122,41 +1165,7 @@ def run_trace(args):
         print(json.dumps(out))
         return
 
-    def st(x):
-        x = np.asarray(x, dtype=np.float64)
-        return {"median": float(np.median(x)), "mean": float(x.mean()), "p90": float(np.percentile(x, 90))}
-    A0, S1, S2, L = T[0], T[1], T[2], T[3]
-    q = np.arange(lo, hi)
-    out["panel_cta"] = {
-        "period": st(A0[q + 1, 0] - A0[q, 0]),
-        "factor_to_step2_records_sent": st(A0[q, 1] - A0[q, 0]),
-        "step2_records_sent_to_panel_done": st(A0[q, 2] - A0[q, 1]),
-        "wait_for_next_block": st(A0[q, 3] - A0[q, 2]),
-        "block_in_to_next_panel_start": st(A0[q + 1, 0] - A0[q, 3]),
-    }
-    for k in range(4):
-        out["panel_cta"][f"step{k}_start_to_barrier"] = st(A0[q, 5 + 3 * k] - A0[q, 4 + 3 * k])
-        out["panel_cta"][f"step{k}_barrier_to_records_sent"] = st(A0[q, 6 + 3 * k] - A0[q, 5 + 3 * k])
-    out["panel_cta"]["panel_start_to_step0_start"] = st(A0[q, 4] - A0[q, 0])
-    # streamer 1 applies panel q's steps 0..2 to block q+1; its last records are step 2's
-    out["streamer1"] = {
-        "block_in_to_first_records": st(S1[q, 1] - S1[q, 0]),
-        "last_records_wait_starts_after_sent": st(S1[q, 2] - A0[q, 1]),
-        "last_records_seen_after_sent": st(S1[q, 3] - A0[q, 1]),
-        "last_step_and_band_send": st(S1[q, 4] - S1[q, 3]),
-        "band_sent_to_panel_cta_has_block": st(A0[q, 3] - S1[q, 4]),
-    }
-    out["streamer2"] = {
-        "block_in_to_first_records": st(S2[q, 1] - S2[q, 0]),
-        "last_records_seen_after_panel_cta_done": st(S2[q, 3] - A0[q, 2]),
-        "band_sent_to_streamer1_block_in": st(S1[q + 1, 0] - S2[q, 4]),
-    }
-    bq = q[L[q, 0] > 0]
-    out["loader_wait_for_hand_over"] = st(L[bq, 1] - L[bq, 0]) if bq.size else None
-    # the supply path: panel b-5 done on A -> its update CTA has applied it and handed block b
-    # over (the loader sees the flag)
-    bs = bq[bq >= lo + 5]
-    out["panel_done_to_hand_over_seen"] = st(L[bs, 1] - A0[bs - 5, 2]) if bs.size else None
+    out.update(trace_summary(T, lo, hi))
     print(json.dumps(out))
 
 
