@@ -192,4 +192,29 @@ __host__ __device__ __forceinline__ double div_known(double x, double d, double 
   return q;
 }
 
+// The back substitution's quotient with the reference-BLAS zero test: x / d for a
+// nonzero x (div_known), x itself for a zero x (no division, its sign kept).  The
+// four-operation path is computed without a branch on x; a zero x fails its
+// exponent-range test and takes the (rare) fallback.
+__host__ __device__ __forceinline__ double div_known_nz(double x, double d, double yh, double yl, bool d_ok) {
+  const int ex = dexp(x), ed = dexp(d);
+  const bool ok = d_ok && ex >= 64 && ex <= 1983 && ex - ed <= 900 && ed - ex <= 900;
+  const double t = x * yl;
+  double q = fma(x, yh, t);
+  const double r = fma(-q, d, x);
+  q = fma(r, yh, q);
+  if (!ok) {
+    if (x != 0.0) {
+#ifdef __CUDA_ARCH__
+      q = div_division(x, d);
+#else
+      q = x / d;
+#endif
+    } else {
+      q = x;
+    }
+  }
+  return q;
+}
+
 }  // namespace bandlu

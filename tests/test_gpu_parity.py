@@ -350,11 +350,13 @@ def assert_same_solution(got, ref):
         raise AssertionError(f"solution not bit-identical first at {tuple(d)}: {got[tuple(d)]!r} vs {ref[tuple(d)]!r}")
 
 
-# windows of 1, 2, 4, 8 and 16 registers per lane, and a CTA with a shared-memory ring (kl+ku+1 > 512,
-# n > ring: the refills)
+# one-warp windows of 1, 2 and 4 registers per lane (kl+ku+1 <= 128); above, the CTA-wide window:
+# 256 threads with one register (kw+33 <= 256), 512 threads with one or two, n below and far above
+# the window (the refills), a sweep of each size in one solve
 @pytest.mark.parametrize("n,kl,ku,nrhs", [(1, 0, 0, 1), (2, 1, 0, 1), (17, 3, 5, 3), (300, 2, 2, 1), (512, 3, 3, 2),
                                           (1000, 16, 16, 5), (700, 0, 12, 1), (700, 12, 0, 1), (600, 40, 40, 2),
-                                          (500, 60, 60, 1), (400, 100, 150, 1), (350, 200, 250, 1),
+                                          (500, 60, 60, 1), (100, 60, 80, 1), (900, 64, 100, 2), (1300, 90, 120, 1),
+                                          (400, 100, 150, 1), (350, 200, 250, 1),
                                           (250, 300, 300, 1), (3000, 300, 300, 2), (2100, 7, 600, 1)])
 def test_gbtrs_matches_oracle(n, kl, ku, nrhs):
     A = banded(n, kl, ku, seed=3 * n + kl + ku, dist="normal").numpy()
