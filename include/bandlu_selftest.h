@@ -33,6 +33,11 @@ int bandlu_selftest_rcp_device(const double *x, double *y, int64_t n, int use_di
  * the host.  x, d and q are HOST arrays of n doubles. */
 void bandlu_selftest_div_host(const double *x, const double *d, double *q, int64_t n);
 
+/* The back substitution's quotient with its zero test, on the host: q[i] = x[i]
+ * for a zero x[i] (either sign: no division, the sign kept), else x[i] / d[i]
+ * with the known-divisor division.  x, d and q are HOST arrays of n doubles. */
+void bandlu_selftest_div_nz_host(const double *x, const double *d, double *q, int64_t n);
+
 /* q[i] = x[i] / d[i] on the device: the library's known-divisor division
  * (use_division == 0) or the compiler's double division (use_division != 0).
  * x, d and q are DEVICE arrays of n doubles; asynchronous on `stream`.

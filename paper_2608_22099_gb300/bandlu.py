@@ -86,6 +86,8 @@ def load():
         lib.bandlu_selftest_rcp_device.restype = ctypes.c_int
         lib.bandlu_selftest_div_host.argtypes = [vp, vp, vp, i64]
         lib.bandlu_selftest_div_host.restype = None
+        lib.bandlu_selftest_div_nz_host.argtypes = [vp, vp, vp, i64]
+        lib.bandlu_selftest_div_nz_host.restype = None
         lib.bandlu_selftest_div_device.argtypes = [vp, vp, vp, i64, i32, vp]
         lib.bandlu_selftest_div_device.restype = ctypes.c_int
         lib.bandlu_peak_dfma.argtypes = [vp, i32, i32, i32, i32, vp]
@@ -249,6 +251,11 @@ def bandlu_selftest_rcp_device(x, y, n: int, use_division: int, stream=None) -> 
 def bandlu_selftest_div_host(x, d, q, n: int) -> None:
     """Self-test hook: the library's known-divisor division on the host (host buffers of n doubles)."""
     load().bandlu_selftest_div_host(_ptr_host(x), _ptr_host(d), _ptr_host(q), n)
+
+
+def bandlu_selftest_div_nz_host(x, d, q, n: int) -> None:
+    """Self-test hook: the back substitution's quotient with its zero test, on the host."""
+    load().bandlu_selftest_div_nz_host(_ptr_host(x), _ptr_host(d), _ptr_host(q), n)
 
 
 def bandlu_selftest_div_device(x, d, q, n: int, use_division: int, stream=None) -> int:

@@ -1,7 +1,8 @@
 // selftest.cu -- self-test hooks (declared in include/bandlu_selftest.h): the
 // integer-pipe reciprocal used on the pivot chain and the known-divisor division
 // of the back substitution, callable on the host and on the device so tests can
-// compare them bit for bit with IEEE division.
+// compare them bit for bit with IEEE division (and the quotient with its zero test
+// on the host).
 #include "bandlu_selftest.h"
 #include "common.cuh"
 #include "rcp.cuh"
@@ -38,6 +39,15 @@ void bandlu_selftest_div_host(const double *x, const double *d, double *q, int64
     bool ok;
     bandlu::div_known_prep(d[i], &yh, &yl, &ok);
     q[i] = bandlu::div_known(x[i], d[i], yh, yl, ok);
+  }
+}
+
+void bandlu_selftest_div_nz_host(const double *x, const double *d, double *q, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) {
+    double yh, yl;
+    bool ok;
+    bandlu::div_known_prep(d[i], &yh, &yl, &ok);
+    q[i] = bandlu::div_known_nz(x[i], d[i], yh, yl, ok);
   }
 }
 

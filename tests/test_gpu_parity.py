@@ -352,12 +352,13 @@ def assert_same_solution(got, ref):
 
 # one-warp windows of 1, 2 and 4 registers per lane (kl+ku+1 <= 128); above, the CTA-wide window:
 # 256 threads with one register (kw+33 <= 256), 512 threads with one or two, n below and far above
-# the window (the refills), a sweep of each size in one solve
+# the window (the refills), a sweep of each size in one solve; kl+ku > 991: the shared-memory ring
 @pytest.mark.parametrize("n,kl,ku,nrhs", [(1, 0, 0, 1), (2, 1, 0, 1), (17, 3, 5, 3), (300, 2, 2, 1), (512, 3, 3, 2),
                                           (1000, 16, 16, 5), (700, 0, 12, 1), (700, 12, 0, 1), (600, 40, 40, 2),
                                           (500, 60, 60, 1), (100, 60, 80, 1), (900, 64, 100, 2), (1300, 90, 120, 1),
                                           (400, 100, 150, 1), (350, 200, 250, 1),
-                                          (250, 300, 300, 1), (3000, 300, 300, 2), (2100, 7, 600, 1)])
+                                          (250, 300, 300, 1), (3000, 300, 300, 2), (2100, 7, 600, 1),
+                                          (1500, 100, 900, 1)])
 def test_gbtrs_matches_oracle(n, kl, ku, nrhs):
     A = banded(n, kl, ku, seed=3 * n + kl + ku, dist="normal").numpy()
     ABf, ipiv, info, _ = oracle.gbtrf(oracle.dense_to_band(A, kl, ku), kl, ku)
@@ -367,8 +368,8 @@ def test_gbtrs_matches_oracle(n, kl, ku, nrhs):
     assert_same_solution(gbtrs_gpu(ABf, ipiv, kl, ku, B), ref)
 
 
-def test_gbtrs_zero_right_hand_sides_and_singular_factor():
-    n, kl, ku = 400, 5, 4
+@pytest.mark.parametrize("n,kl,ku", [(400, 5, 4), (600, 70, 90), (700, 200, 250)])
+def test_gbtrs_zero_right_hand_sides_and_singular_factor(n, kl, ku):
     A = banded(n, kl, ku, seed=77).numpy()
     ABf, ipiv, info, _ = oracle.gbtrf(oracle.dense_to_band(A, kl, ku), kl, ku)
     B = np.zeros((3, n))

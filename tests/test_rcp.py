@@ -102,6 +102,24 @@ def test_known_divisor_division_host_copy_is_ieee_division():
     assert not bad.any(), list(zip(x[bad][:5], d[bad][:5]))
 
 
+def test_quotient_with_zero_test_host_copy():
+    """The back substitution's quotient (the CTA-wide solve): a zero dividend of either sign is
+    kept as it is (the reference BLAS skips the division), which x / d would not do for a
+    negative d; every other dividend is divided exactly as IEEE division does."""
+    x, d = division_pairs(600_000, 23)
+    x[:4000] = 0.0
+    x[4000:8000] = -0.0
+    d[:2000] = -np.abs(d[:2000])                      # +0 / negative and -0 / positive would flip
+    d[6000:7000] = np.abs(d[6000:7000])
+    q = np.empty_like(x)
+    bandlu.bandlu_selftest_div_nz_host(x, d, q, x.size)
+    with np.errstate(all="ignore"):
+        ref = np.where(x != 0.0, x / d, x)
+    bad = ~same_bits(q, ref)
+    assert not bad.any(), list(zip(x[bad][:5], d[bad][:5]))
+    assert np.signbit(q[:2000]).sum() == 0 and np.signbit(q[4000:8000]).all()
+
+
 @pytest.mark.gpu
 def test_known_divisor_division_device_is_ieee_division():
     import torch
