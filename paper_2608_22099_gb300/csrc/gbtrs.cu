@@ -7,9 +7,10 @@
 //            j+1..j+kl take fma(-l, b_j, .);
 //   backward j = n-1..0: if b_j != 0, b_j = b_j / u_jj and rows j-kv..j-1 take
 //            fma(-b_j, u, .).
-// One warp per right-hand side keeps the active part of b in registers, in a
-// window that rotates with the steps (trwin.cuh); the division by u_jj uses a
-// two-term reciprocal formed ahead of time, 32 diagonal entries at once
+// The active part of b stays in registers, in a window that rotates with the
+// steps: one warp per right-hand side up to kl+ku+1 = 128 rows (trwin.cuh), a
+// CTA of 256 or 512 threads per right-hand side and sweep above (cta_sweep).
+// The division by u_jj uses a two-term reciprocal formed ahead of time
 // (div_known: four dependent FP64 operations instead of a full division).  The
 // same operations in the same order as the oracle, so the solution is
 // bit-identical to it.  Interchanges outside j..j+kl (not produced by gbtrf)
@@ -255,6 +256,7 @@ __device__ __forceinline__ void cta_sweep(double *b, int n, int kw, const Src &s
     if (warp == bw(1)) nd = dload(1);
   }
   // what step k reads, published by the owners (slot (k & 1) of pub: value, partner)
+  // step 0's values, before the loop (inside it, each step publishes for the next)
   auto publish = [&](int k, int s) {
     if (kDiv) {
       if (warp == (owner(k) >> 5) && lane == (k & 31)) {
@@ -497,9 +499,9 @@ int launch_window(int n, int kl, int ku, int nrhs, const double *AB, int ldab, c
 }
 
 // Windows up to this many rows take the one-warp register window, wider ones the
-// CTA-wide window (measured on GB300: the one-warp window is faster up to kl+ku+1 =
-// 73, the CTA 1.4x faster at 129 and 2.2x at 451; BANDLU_GBTRS_CTA_ABOVE=<rows>
-// moves the switch, for measurement).
+// CTA-wide window (measured on GB300, n = 16384: the CTA 1.9x faster at kl+ku+1 =
+// 129 and 2.4x at 451; the one-warp window faster at 65 and 73 than the first,
+// 512-thread CTA; BANDLU_GBTRS_CTA_ABOVE=<rows> moves the switch, for measurement).
 long long cta_min_window() {
   static const long long w = [] {
     const char *v = std::getenv("BANDLU_GBTRS_CTA_ABOVE");
