@@ -168,11 +168,13 @@ __global__ void __launch_bounds__(256) k_gbtrs_cta(int n, int kl, int ku, int WS
 // barrier.
 //   Before it, the owners of what step k reads publish it in shared memory:
 //   forward, the value at position k and the one it is interchanged with;
-//   backward, the quotient x_k, which its owner forms (div_known, the divisor's
-//   two-term reciprocal ready) right after applying step k-1 to that position,
-//   before the other registers of its warp.
+//   backward, the quotient x_k, which its owner forms (div_known_nz, the
+//   divisor's two-term reciprocal ready) right after applying step k-1 to that
+//   position, before the other registers of its warp.
 //   After it, every thread applies step k to the positions k+1..k+mk it holds:
-//   one FP64 instruction per warp register that holds any of them.
+//   one FP64 instruction per warp register that holds any of them, with the
+//   zero test as a select after it.  Everything that does not depend on the
+//   step's value is computed before the barrier.
 // The warp whose 32 positions a block of 32 steps eliminates refills them at the
 // block's end with the positions W further on (W >= kw + 33, so a refilled
 // position is first updated after that block).  The divisors of a block are read
@@ -255,8 +257,9 @@ __device__ __forceinline__ void cta_sweep(double *b, int n, int kw, const Src &s
     }
     if (warp == bw(1)) nd = dload(1);
   }
-  // what step k reads, published by the owners (slot (k & 1) of pub: value, partner)
-  // step 0's values, before the loop (inside it, each step publishes for the next)
+  // What step k reads, published by its owners into slot k & 1 of pub (value,
+  // interchange partner): here step 0's, before the loop; inside it, each step
+  // publishes for the next.
   auto publish = [&](int k, int s) {
     if (kDiv) {
       if (warp == (owner(k) >> 5) && lane == (k & 31)) {
